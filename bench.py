@@ -1,0 +1,404 @@
+#!/usr/bin/env python3
+"""Benchmark of one DARD denoising step on GB300: state-masked attention + scoring.
+
+A step is one pass of the whole hot path over one batch of synthetic input: the masked
+attention of one layer (dard_step_attention) followed by confidence scoring and the state
+transition (dard_score_and_transition, two PDL-chained kernels). The workload is the
+8B-class layer: 32 heads MHA, head_dim 128, prompt 512, generation 256 in blocks of 32,
+current block 3, shadow copy of the current block (800 rows), logits 32 x 126464 bf16.
+
+Timing: CUDA graphs of 16 consecutive steps, each on its own input set (16 sets, 675 MB,
+more than 4x the 129 MB L2), replayed back to back between CUDA events; per-kernel averages
+from graphs of the same 16 launches of one kernel. e2e: the same step through the C ABI
+from pinned host buffers, host->device copies of the inputs and device->host copies of the
+results inside the timed region.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "DARD step µs at 8B shape: masked-attn TFLOP/s (% peak), score GB/s (% HBM)"
+NSETS = 16
+WORKLOAD_DESC = ("8B-class layer: 32 heads MHA, head_dim 128, prompt 512 + generation 256 in "
+                 "blocks of 32, current block 3 (b0=608, N=768), states 16/8/8 M/C/U, shadow "
+                 "copy of the current block (800 rows), Q/K/V bf16 N(0,1)/sqrt(128); logits "
+                 "2 x 32 x 126464 bf16 N(0,3), +6 planted on 40% of rows")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--layout", default="paper", choices=["paper", "candidates"])
+    ap.add_argument("--e2e-steps", type=int, default=300)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------------------ clocks
+CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockMonitor:
+    """nvidia-smi sampling every 100 ms while the timed region runs."""
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={CLOCK_FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r for r in csv.reader(io.StringIO(self.f.read())) if len(r) >= 9]
+        os.unlink(self.f.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ helpers
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d["bf16_tflops"], "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def traffic_for(kernel: str, source: str, per_launch_units: float):
+    """DRAM bytes per launch from profiles/traffic.txt, if recorded for this source hash."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    digest = hashlib.sha256(open(os.path.join(ROOT, source), "rb").read()).hexdigest()[:16]
+    for line in open(path):
+        parts = line.split()
+        if len(parts) >= 3 and parts[0] == kernel and parts[1] == digest:
+            return float(parts[2]) * per_launch_units
+    return None
+
+
+def oracle_step(wl, rows=None):
+    """One oracle pass over the workload's first sequence: mask + attention (all heads) for
+    `rows` query rows (all when None) and scoring of the whole block. Returns
+    (attention seconds, scoring seconds)."""
+    import numpy as np
+    import oracle as orc
+    s = wl.seqs[0]
+    lay = orc.SeqLayout(s.n_orig, s.block_start, s.state, s.prev_conf, s.shadow_src)
+    t0 = time.perf_counter()
+    mask = orc.attention_mask(lay, rows=rows)
+    orc.masked_attention(wl.q[0], wl.k[0], wl.v[0], mask, rows=rows)
+    t1 = time.perf_counter()
+    orc.score_block(wl.logits_x, wl.logits_s, s.state, float(np.float32(wl.tau_c)),
+                    float(np.float32(wl.tau_u)), float(np.float32(wl.lam)),
+                    float(np.float32(wl.p0)))
+    t2 = time.perf_counter()
+    return t1 - t0, t2 - t1
+
+
+def blas_threads() -> int:
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    return os.cpu_count() or 1
+
+
+def cpu_baseline(wl, seconds: float) -> dict:
+    """The oracle as it stands, timed on full steps of the workload for about `seconds`."""
+    att, sc, n = 0.0, 0.0, 0
+    t_end = time.perf_counter() + seconds
+    while time.perf_counter() < t_end or n == 0:
+        a, s = oracle_step(wl)
+        att, sc, n = att + a, sc + s, n + 1
+    per = (att + sc) / n
+    return {"value": per * 1e6, "unit": "µs", "cores": blas_threads(), "kind": "oracle",
+            "sample": f"{n} full 8B-class steps (mask + fp64 attention of all 800 rows x 32 "
+                      f"heads + scoring of the 32-row block); BLAS matmuls on {blas_threads()} "
+                      f"threads, the rest of numpy on 1"}
+
+
+# ------------------------------------------------------------------------------ reference arm
+def run_reference(args, rank: int):
+    if rank != 0:
+        return
+    import numpy as np
+    from paper_2608_26574_gb300 import workloads as W
+    wl = W.make("8b", layout=args.layout)
+    rows_total = wl.seqs[0].rows
+    # calibrate the per-row cost on one full pass (counted as a warm-up step)
+    a_full, s_full = oracle_step(wl)
+    budget = 150.0
+    per_step = budget / max(1, args.steps + args.warmup)
+    rows_per_step = int(max(1, min(rows_total, per_step / max(a_full / rows_total, 1e-9))))
+    score_every = int(max(1, math.ceil(s_full / max(per_step * 0.3, 1e-9))))
+    att_t, att_rows, sc_t, sc_n = 0.0, 0, 0.0, 0
+    cursor = 0
+    for step in range(args.warmup + args.steps):
+        rows = (cursor + np.arange(rows_per_step)) % rows_total
+        cursor = (cursor + rows_per_step) % rows_total
+        import oracle as orc
+        s = wl.seqs[0]
+        lay = orc.SeqLayout(s.n_orig, s.block_start, s.state, s.prev_conf, s.shadow_src)
+        t0 = time.perf_counter()
+        mask = orc.attention_mask(lay, rows=rows)
+        orc.masked_attention(wl.q[0], wl.k[0], wl.v[0], mask, rows=rows)
+        t1 = time.perf_counter()
+        ts = 0.0
+        if step % score_every == 0:
+            orc.score_block(wl.logits_x, wl.logits_s, s.state, float(np.float32(wl.tau_c)),
+                            float(np.float32(wl.tau_u)), float(np.float32(wl.lam)),
+                            float(np.float32(wl.p0)))
+            ts = time.perf_counter() - t1
+        if step >= args.warmup:
+            att_t += t1 - t0
+            att_rows += rows_per_step
+            if step % score_every == 0:
+                sc_t += ts
+                sc_n += 1
+    if sc_n == 0:
+        sc_t, sc_n = s_full, 1
+    per_step_us = (att_t / max(att_rows, 1) * rows_total + sc_t / sc_n) * 1e6
+    sample = (f"each step: mask + fp64 attention of {rows_per_step} of {rows_total} query rows "
+              f"(all 32 heads); the 32-row scoring block every {score_every} steps; value "
+              f"extrapolated to a full step by rows")
+    line = {"impl": "reference", "metric": METRIC, "value": per_step_us, "unit": "µs",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": per_step_us / 1e3, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC, "layout": args.layout},
+            "cpu_baseline": {"value": per_step_us, "unit": "µs", "cores": blas_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": per_step_us, "unit": "µs", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------ our arm
+def run_ours(args, rank: int, world: int):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_26574_gb300 import binding as Bd
+    from paper_2608_26574_gb300 import build as Bu
+    from paper_2608_26574_gb300 import workloads as W
+    from paper_2608_26574_gb300.device import DeviceStep
+
+    Bu.build()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    wl = W.make("8b", layout=args.layout)
+    ds = DeviceStep(wl, device=dev)
+    q0, k0, v0, _ = ds.layers[0]
+    sets = []
+    for _ in range(NSETS):
+        sets.append(dict(q=q0.clone(), k=k0.clone(), v=v0.clone(), o=torch.empty_like(q0),
+                         lx=ds.lx.clone(), ls=ds.ls.clone()))
+    meta = (ds.n_orig, ds.block_start, ds.block_len, ds.shadow_len)
+
+    def attn(s):
+        Bd.dard_step_attention(s["q"], s["k"], s["v"], s["o"], *meta, ds.state, ds.prev_conf,
+                               ds.shadow_src, status=ds.status)
+
+    def score(s):
+        Bd.dard_score_and_transition(s["lx"], s["ls"], ds.block_len, ds.state, wl.tau_c,
+                                     wl.tau_u, wl.lam, wl.p0, ds.conf, ds.token, ds.state_out,
+                                     ds.workspace, w_out=ds.w_out, counts=ds.counts,
+                                     status=ds.status)
+
+    for i in range(max(3, args.warmup)):
+        attn(sets[i % NSETS])
+        score(sets[i % NSETS])
+    torch.cuda.synchronize()
+
+    def capture(fn, n):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(n):
+                fn(sets[i % NSETS])
+        return g
+
+    step = lambda s: (attn(s), score(s))  # noqa: E731
+    g_step = capture(step, NSETS)
+    tail = args.steps % NSETS
+    g_tail = capture(step, tail) if tail else None
+    g_attn = capture(attn, NSETS)
+    g_score = capture(score, NSETS)
+    for g in (g_step, g_attn, g_score):
+        g.replay()
+    torch.cuda.synchronize()
+
+    def timed(g, reps, g_extra=None):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            g.replay()
+        if g_extra is not None:
+            g_extra.replay()
+        e1.record()
+        e1.synchronize()
+        return e0.elapsed_time(e1)
+
+    mon = ClockMonitor(local)
+    mon.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ms = timed(g_step, args.steps // NSETS, g_tail)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = mon.stop()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / args.steps
+
+    # per-kernel averages (same launches, one kernel per graph)
+    reps = max(4, min(400, int(0.25 / max(ms_per_step / 1e3, 1e-6) / NSETS)))
+    attn_us = timed(g_attn, reps) * 1e3 / (reps * NSETS)
+    score_us = timed(g_score, reps) * 1e3 / (reps * NSETS)
+    status = int(ds.status.item())
+
+    # e2e through the C ABI from pinned host buffers
+    host_in = {k: sets[0][k].cpu().pin_memory() for k in ("q", "k", "v", "lx", "ls")}
+    host_meta = {"state": ds.state.cpu().pin_memory(), "prev_conf": ds.prev_conf.cpu().pin_memory(),
+                 "shadow_src": ds.shadow_src.cpu().pin_memory()}
+    outs = {"conf": ds.conf, "token": ds.token, "state_out": ds.state_out, "counts": ds.counts}
+    host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in outs.items()}
+    d_meta = {"state": ds.state, "prev_conf": ds.prev_conf, "shadow_src": ds.shadow_src}
+    h2d = sum(t.numel() * t.element_size() for t in list(host_in.values()) + list(host_meta.values()))
+    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+    s0 = sets[0]
+
+    def e2e_step():
+        for k, t in host_in.items():
+            s0[k].copy_(t, non_blocking=True)
+        for k, t in host_meta.items():
+            d_meta[k].copy_(t, non_blocking=True)
+        attn(s0)
+        score(s0)
+        for k, t in outs.items():
+            host_out[k].copy_(t, non_blocking=True)
+
+    for _ in range(5):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record()
+    e1.synchronize()
+    e2e_us = e0.elapsed_time(e1) * 1e3 / args.e2e_steps
+
+    if rank != 0:
+        return
+    hbm, bf16, peak_kind = peaks()
+    flops = W.attention_flops(wl)
+    sbytes = W.scoring_bytes(wl)
+    att_tflops = flops / (attn_us * 1e-6) / 1e12
+    sc_gbs = sbytes / (score_us * 1e-6) / 1e9
+    line = {
+        "metric": METRIC, "value": ms_per_step * 1e3, "unit": "µs", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_DESC, "layout": args.layout,
+                   "l2": f"{NSETS} rotating input sets (~675 MB) > 4x L2",
+                   "parallelism": f"replicas x{world}", "timing": "CUDA-graph replays"},
+        "roofline": {"bound": "tensor", "kernel": "attn_tc<128>", "achieved": att_tflops,
+                     "peak": bf16, "unit": "TFLOP/s", "frac": att_tflops / bf16,
+                     "peak_kind": f"{peak_kind} bf16 burst",
+                     "traffic": traffic_for("attn_tc", "paper_2608_26574_gb300/csrc/dard_attention.cu", 1.0),
+                     "algorithmic_flops_per_launch": flops},
+        "kernels": {"attention_us": attn_us, "attention_tflops": att_tflops,
+                    "attention_frac_bf16": att_tflops / bf16, "scoring_us": score_us,
+                    "scoring_gbs": sc_gbs, "scoring_frac_hbm": sc_gbs / hbm,
+                    "scoring_frac_8tbs": sc_gbs / 8000.0, "scoring_bytes_per_call": sbytes},
+        "clocks": clocks,
+        "e2e": {"value": e2e_us, "unit": "µs", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": args.steps * 3,
+        "status_word": status,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

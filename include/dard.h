@@ -1,0 +1,179 @@
+/*
+ * dard.h - C ABI of the GB300 (sm_103a) DARD step library, libdard.so.
+ *
+ * DARD (Dependency-Aware Revocable Decoding, arXiv 2608.26574) adds two pieces of compute
+ * to every denoising step of a diffusion LLM:
+ *
+ *   dard_step_attention        bidirectional softmax attention over the augmented sequence
+ *                              x~_t = (x_t; s_t) under the state-specific mask of Sec. 3
+ *                              (Eq. 2, Eq. 3 and query blocks 1-6 of Sec. 3.2), one layer;
+ *   dard_score_and_transition  vocabulary-wide confidence and argmax (Eq. 1), verification
+ *                              outcomes and guidance weights (Eq. 5, Eq. 6), logit mixing
+ *                              (Eq. 7) and the three-state transition (Eq. 8), in the order
+ *                              of Algorithm 1.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers named "device" are CUDA device memory owned by the caller; pointers named
+ *     "host" are ordinary host memory owned by the caller and read during the call only.
+ *   - Every call is asynchronous on the given stream; nothing is synchronised.
+ *   - The library never allocates memory. Scratch space is passed in by the caller.
+ *   - Argument and shape errors are detected on the host and returned before any launch;
+ *     nothing is launched when a call returns an error. A failed launch returns
+ *     DARD_ERR_CUDA (the CUDA error string is available from dard_last_error()).
+ *   - Problems found only on the device (a state byte above 2, a shadow row that points
+ *     outside its block, a row whose softmax normaliser is not finite) never trap: they set
+ *     bits of the optional device status word (DARD_STATUS_*) and the affected outputs follow
+ *     the documented fallback.
+ *
+ * Sequence layout (per sequence i of a ragged batch, everything stored back to back):
+ *   rows      N_i original rows (prompt + full generation length, positions 0..N_i-1),
+ *             then S_i shadow rows. Row N_i + k is the shadow copy s^j, j = shadow_src[k].
+ *   block     positions [b0_i, b0_i + B_i) are the block being decoded. Positions before
+ *             it are decoded context (state U); positions after it are still masked
+ *             (state M) and have no shadow row.
+ *   states    one byte per block position: 0 = M (masked), 1 = C (candidate),
+ *             2 = U (unmasked), the three states of Sec. 3.2.
+ */
+#ifndef DARD_H_
+#define DARD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DARD_OK = 0,
+  DARD_ERR_NULL = 1,         /* a required pointer is NULL                              */
+  DARD_ERR_SHAPE = 2,        /* inconsistent sizes / offsets                            */
+  DARD_ERR_VALUE = 3,        /* a parameter out of its range (tau, lambda, p0, scale)   */
+  DARD_ERR_UNSUPPORTED = 4,  /* valid but not implemented (e.g. head_dim not 64 or 128) */
+  DARD_ERR_CUDA = 5,         /* a CUDA runtime call failed                              */
+  DARD_ERR_ALIGN = 6,        /* a pointer or stride breaks the alignment rule           */
+  DARD_ERR_WORKSPACE = 7     /* workspace missing or smaller than required              */
+} dard_status;
+
+typedef enum { DARD_F32 = 0, DARD_BF16 = 1 } dard_dtype;
+
+/* Bits of the optional device status word (OR-ed in, never cleared by the library). */
+#define DARD_STATUS_BAD_STATE 0x1u     /* a state byte > 2 (treated as M)                    */
+#define DARD_STATUS_BAD_SHADOW 0x2u    /* shadow_src outside its block or repeated (row
+                                          treated as a masked-out key and left unwritten)    */
+#define DARD_STATUS_INVALID_ROW 0x4u   /* softmax normaliser not finite or zero (NaN, +inf or
+                                          all -inf logits): conf 0, token -1, state M        */
+#define DARD_STATUS_TIMEOUT 0x8u       /* a bounded in-kernel wait gave up (the launch's
+                                          outputs are incomplete)                             */
+
+#define DARD_MAX_SEQS 256       /* sequences per call                                     */
+#define DARD_MAX_BLOCK 128      /* block length B_i                                       */
+
+/* ------------------------------------------------------------------------------------- *
+ * Masked attention (Sec. 3.1 Eq. 2; Sec. 3.2 query blocks 1-6 and Eq. 3).
+ *
+ * For every sequence, head h and row r:
+ *     O[r,h,:] = sum_j softmax_j(scale * <Q[r,h,:], K[key(r,j),g,:]>) V[key(r,j),g,:]
+ * where j runs over the N_i original positions, key(r,j) is the row of x^j or of s^j as
+ * the mask selects (exactly one per position, Eq. 2), and g = h / (hq / hkv) (grouped-query
+ * heads share a key/value head). The mask is built inside the kernel from the state vector
+ * and prev_conf; no L x L tensor exists anywhere. Selection rule (q = query copy):
+ *   key j state U : x^j, except a shadow query s^i takes s^i for j = i;
+ *   key j state M : x^j for original queries of M positions, s^j for every other query;
+ *   key j state C : original query of an M position       -> x^j
+ *                   query of a C position i (x or s)      -> x^j if c_i <= c_j, else s^j
+ *                                                            (a shadow query takes s^i at j=i)
+ *                   query of a U position, or s^i of an M -> s^j
+ *   and x^j whenever j has no shadow row (positions outside the block, or a block position
+ *   the caller gave no shadow row). Out-of-block queries are original queries of U (before
+ *   the block) or M (after it) positions.
+ * Arithmetic: bf16 operands on the tcgen05 tensor cores with fp32 accumulation and an fp32
+ * online softmax (dtype BF16); fp32 CUDA cores throughout (dtype F32).
+ * ------------------------------------------------------------------------------------- */
+typedef struct {
+  const void* q;             /* device [total_rows, hq,  head_dim] row-major              */
+  const void* k;             /* device [total_rows, hkv, head_dim]                        */
+  const void* v;             /* device [total_rows, hkv, head_dim]                        */
+  void* o;                   /* device [total_rows, hq,  head_dim], same dtype as q       */
+  int32_t dtype;             /* dard_dtype of q, k, v and o                                */
+  int32_t hq, hkv;           /* query heads, key/value heads; hq % hkv == 0                */
+  int32_t head_dim;          /* 64 or 128                                                  */
+  int32_t num_seqs;          /* 1 .. DARD_MAX_SEQS                                         */
+  const int32_t* n_orig;     /* host [num_seqs] N_i >= 1                                   */
+  const int32_t* block_start;/* host [num_seqs] b0_i, 0 <= b0_i, b0_i + B_i <= N_i         */
+  const int32_t* block_len;  /* host [num_seqs] B_i in 0 .. DARD_MAX_BLOCK                 */
+  const int32_t* shadow_len; /* host [num_seqs] S_i in 0 .. B_i                            */
+  const uint8_t* state;      /* device [sum B_i] states of block positions, seq by seq     */
+  const float* prev_conf;    /* device [sum B_i] c_{t-1} of block positions (Eq. 3 order)  */
+  const int32_t* shadow_src; /* device [sum S_i] original position of each shadow row,
+                                in [b0_i, b0_i + B_i), distinct within a sequence          */
+  float scale;               /* softmax scale; 0 means 1/sqrt(head_dim)                    */
+  uint32_t* status;          /* optional device word, DARD_STATUS_* bits OR-ed in          */
+} dard_attn_args;
+
+/* Rows are total_rows = sum_i (N_i + S_i). q, k, v, o must be 16-byte aligned; with dtype
+ * BF16 the tensor-core kernel runs (head_dim 64 or 128), with F32 the CUDA-core kernel.
+ * Errors: DARD_ERR_NULL, _SHAPE, _VALUE (scale < 0 or not finite), _UNSUPPORTED,
+ * _ALIGN, _CUDA. */
+dard_status dard_step_attention(const dard_attn_args* args, void* stream /* cudaStream_t */);
+
+/* ------------------------------------------------------------------------------------- *
+ * Confidence scoring and state transition (Eq. 1, Eq. 5-8, Algorithm 1).
+ *
+ * Rows are the block positions of all sequences, seq by seq (sum B_i rows). For row i of a
+ * sequence with incoming state s_i:
+ *   s_i in {C, U}: (c_i, x^_i) = (max softmax, argmax) of logits_s row i          (Eq. 1)
+ *   then every C row that moves to U joins P, every C row that moves to M joins D (Eq. 8);
+ *   s_i = M: P_i = sum_{j in P} lambda^|i-j|, D_i likewise over D                  (Eq. 5)
+ *            w_i = (P_i + p0) / (P_i + D_i + p0)                                  (Eq. 6)
+ *            mix = ls + w_i (lx - ls), each operation rounded to fp32              (Eq. 7)
+ *            (c_i, x^_i) = (max softmax, argmax) of mix
+ *   new state: c <= tau_c -> M, c <= tau_u -> C, else U                            (Eq. 8)
+ * Argmax ties go to the lowest index. Softmax sums accumulate in fp32; w in fp64.
+ * Invalid rows (normaliser not finite or 0): conf 0, token -1, state M, status bit.
+ * ------------------------------------------------------------------------------------- */
+typedef struct {
+  const void* logits_x;      /* device [rows, row_stride] logits of the original copies   */
+  const void* logits_s;      /* device [rows, row_stride] logits of the shadow copies     */
+  int32_t dtype;             /* dard_dtype of both logit tensors                           */
+  int32_t vocab;             /* V >= 1                                                     */
+  int64_t row_stride;        /* elements between consecutive rows, >= vocab               */
+  int32_t num_seqs;          /* 1 .. DARD_MAX_SEQS                                         */
+  const int32_t* block_len;  /* host [num_seqs] B_i in 0 .. DARD_MAX_BLOCK                 */
+  const uint8_t* state_in;   /* device [rows] incoming states                              */
+  float tau_c, tau_u;        /* 0 <= tau_c <= tau_u <= 1                                   */
+  float lambda;              /* 0 < lambda < 1 (paper: 0.5^(1/8))                          */
+  float p0;                  /* p0 > 0 (paper: 0.1)                                        */
+  float* conf;               /* device [rows] out: c_t                                     */
+  int32_t* token;            /* device [rows] out: x^_t (or -1 for an invalid row)         */
+  uint8_t* state_out;        /* device [rows] out: state after Eq. 8                       */
+  float* w_out;              /* optional device [rows] out: w for M rows, NaN otherwise    */
+  int32_t* counts;           /* optional device [num_seqs * 3] out: M, C, U counts         */
+  uint32_t* status;          /* optional device word, DARD_STATUS_* bits OR-ed in          */
+  void* workspace;           /* device scratch of dard_score_workspace_size() bytes, zeroed
+                                once by the caller after allocation; every call leaves it
+                                zeroed again. Calls that overlap on the GPU need separate
+                                workspaces.                                                */
+  size_t workspace_bytes;
+} dard_score_args;
+
+/* Bytes of workspace a call with these sizes needs (0 on invalid sizes). */
+size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs);
+
+/* Logits pointers must be 16-byte aligned and row_stride * element size a multiple of 16.
+ * Errors: DARD_ERR_NULL, _SHAPE, _VALUE, _ALIGN, _WORKSPACE, _CUDA. */
+dard_status dard_score_and_transition(const dard_score_args* args, void* stream);
+
+/* Human-readable name of a status code; never NULL. */
+const char* dard_status_string(dard_status s);
+
+/* The message of the last DARD_ERR_CUDA / validation failure on this thread; never NULL. */
+const char* dard_last_error(void);
+
+/* Library version as major * 10000 + minor * 100 + patch. */
+int32_t dard_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DARD_H_ */

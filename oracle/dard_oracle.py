@@ -163,9 +163,10 @@ def sees_shadow_copy(copy: str, i: int, st: np.ndarray, conf: np.ndarray) -> np.
     return out
 
 
-def attention_mask(lay: SeqLayout) -> np.ndarray:
-    """Dense boolean mask over the rows of x~_t: mask[r, kr] is True iff query row r attends
-    key row kr. Row/key order: the N original rows, then the S shadow rows.
+def attention_mask(lay: SeqLayout, rows: np.ndarray | None = None) -> np.ndarray:
+    """Boolean mask over the rows of x~_t: mask[a, kr] is True iff query row rows[a] (every
+    row when ``rows`` is None) attends key row kr. Row/key order: the N original rows, then
+    the S shadow rows.
 
     Eq. 2 holds by construction: for every position j exactly one of x^j and s^j is True.
     Where the rule picks s^j but j has no shadow row, x^j is taken (R3).
@@ -173,14 +174,15 @@ def attention_mask(lay: SeqLayout) -> np.ndarray:
     st = position_states(lay)
     conf = position_conf(lay)
     sh = shadow_row_of(lay)
-    rows, n = lay.rows, lay.n_orig
-    mask = np.zeros((rows, rows), dtype=bool)
+    n = lay.n_orig
+    rows = np.arange(lay.rows) if rows is None else np.asarray(rows)
+    mask = np.zeros((len(rows), lay.rows), dtype=bool)
     j = np.arange(n)
-    for r in range(rows):
-        copy, i = query_identity(lay, r)
+    for a, r in enumerate(rows):
+        copy, i = query_identity(lay, int(r))
         take_s = sees_shadow_copy(copy, i, st, conf) & (sh >= 0)
-        mask[r, j[~take_s]] = True
-        mask[r, sh[take_s]] = True
+        mask[a, j[~take_s]] = True
+        mask[a, sh[take_s]] = True
     return mask
 
 
@@ -191,9 +193,10 @@ def masked_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, mask: np.ndarr
                      scale: float | None = None, rows: np.ndarray | None = None) -> np.ndarray:
     """O[r, h] = sum_kr softmax_kr(scale * <q[r,h], k[kr,g]>, over mask[r]) * v[kr, g].
 
-    q: [R, Hq, d]; k, v: [R, Hkv, d]; mask: [R, R]; g = h // (Hq // Hkv) (grouped-query
-    heads share a key/value head). ``rows`` restricts the query rows computed (for sampled
-    parity at full size). Returns float64 [len(rows), Hq, d].
+    q: [R, Hq, d]; k, v: [R, Hkv, d]; g = h // (Hq // Hkv) (grouped-query heads share a
+    key/value head). ``rows`` restricts the query rows computed (for sampled parity at full
+    size); ``mask`` holds one row per computed query row ([R, R], or [len(rows), R]).
+    Returns float64 [len(rows), Hq, d].
     """
     R, hq, d = q.shape
     hkv = k.shape[1]
@@ -203,15 +206,15 @@ def masked_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, mask: np.ndarr
         scale = 1.0 / math.sqrt(d)  # R8
     if rows is None:
         rows = np.arange(R)
+    assert mask.shape == (len(rows), k.shape[0])
     q64 = q[rows].astype(np.float64)
     k64 = k.astype(np.float64)
     v64 = v.astype(np.float64)
-    sub = mask[rows]
     out = np.empty((len(rows), hq, d), dtype=np.float64)
     for h in range(hq):
         g = h // group
         z = (q64[:, h, :] @ k64[:, g, :].T) * scale
-        z = np.where(sub, z, -np.inf)
+        z = np.where(mask, z, -np.inf)
         z = z - z.max(axis=1, keepdims=True)
         p = np.exp(z)
         p = p / p.sum(axis=1, keepdims=True)

@@ -1,0 +1,543 @@
+// dard_attention.cu - state-masked bidirectional attention of one DARD step (sm_103a).
+//
+// The augmented sequence x~_t = (x_t; s_t) of arXiv 2608.26574 Sec. 3.1 is stored per
+// sequence as N original rows followed by S shadow rows. Every query attends exactly one
+// copy (x^j or s^j) of every original position j (Eq. 2); which copy is decided in-kernel
+// from the block's state vector and c_{t-1} (Sec. 3.2, query blocks 1-6 and Eq. 3). Key
+// tiles that touch neither the current block nor the shadow rows are dense for every query,
+// so the mask is evaluated only on the (at most three) tiles that contain block keys,
+// shadow keys or the ragged end of the sequence.
+//
+// bf16 path (attn_tc): one CTA = 128 query rows of one (sequence, head); 6 warps:
+//   warps 0-3  softmax and epilogue, thread t owns query row t (= TMEM lane t);
+//   warp 4     TMA producer (Q once, then K and V tiles of 128 keys) and TMEM allocator;
+//   warp 5     tcgen05 MMA issuer: S = Q K^T into TMEM, then O += P V with P (bf16) read
+//              from TMEM where the softmax warps wrote it over S.
+// The online softmax keeps a per-row running maximum and rescales O in TMEM only when the
+// maximum grows by more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
+// fp32 path (attn_simt): CUDA-core kernel, one warp per query row, same mask logic.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <climits>
+#include <atomic>
+#include <cmath>
+#include <cstdio>
+#include <mutex>
+#include <numeric>
+#include <vector>
+
+#include "dard_internal.h"
+#include "dard_ptx.cuh"
+
+namespace dard {
+namespace {
+
+constexpr int kBM = 128;  // query rows per CTA
+constexpr int kBN = 128;  // keys per tile
+constexpr int kTcThreads = 192;
+constexpr uint32_t kTmemCols = 256;  // S/P: columns [0,128), O: [128, 128 + D)
+constexpr float kRescaleLog2 = 8.0f;
+
+// Per-CTA copy of the current block: states, confidences and the shadow maps.
+struct BlockInfo {
+  int32_t st[DARD_MAX_BLOCK];
+  float cf[DARD_MAX_BLOCK];
+  int32_t shrow[DARD_MAX_BLOCK];  // block position -> shadow row index k, or -1
+  int32_t shpos[DARD_MAX_BLOCK];  // shadow row index k -> block position, or -1 if invalid
+};
+
+// The query a row stands for: its copy (x or s), its state, c_{t-1}, block position.
+struct RowInfo {
+  int qs;     // 1 for a shadow query s^i
+  int si;     // state of position i
+  float ci;   // c_{t-1} of position i (block positions only)
+  int i;      // block position of i, or -1 outside the block
+  int store;  // 0 for padding rows and invalid shadow rows
+};
+
+__device__ __forceinline__ void sm_bar_sync() {  // warps 0-3 only
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+}
+
+__device__ __forceinline__ void decode_work(const AttnParams& p, int w, int& seq, int& qt,
+                                            int& h) {
+  int lo = 0, hi = p.num_seqs;  // work_prefix[lo] <= w < work_prefix[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (p.work_prefix[mid] <= w) lo = mid; else hi = mid;
+  }
+  seq = p.order[lo];
+  const int local = w - p.work_prefix[lo];
+  h = local % p.hq;
+  qt = local / p.hq;
+}
+
+// Called by the 128 threads of warps 0-3. A repeated shadow position keeps its lowest
+// shadow row; the others, and positions outside the block, are flagged and never used.
+__device__ void load_block_info(const AttnParams& p, const SeqDesc& sd, BlockInfo& bi,
+                                bool report) {
+  const int t = threadIdx.x;
+  bi.shrow[t] = INT_MAX;
+  bi.shpos[t] = -1;
+  if (t < sd.blen) {
+    int s = p.state[sd.blk_off + t];
+    if (s > 2) {
+      if (report && p.status) atomicOr(p.status, DARD_STATUS_BAD_STATE);
+      s = kStateM;
+    }
+    bi.st[t] = s;
+    bi.cf[t] = p.prev_conf[sd.blk_off + t];
+  }
+  int pos = -1;
+  if (t < sd.slen) pos = p.shadow_src[sd.sh_off + t] - sd.b0;
+  const bool in_block = pos >= 0 && pos < sd.blen;
+  sm_bar_sync();
+  if (t < sd.slen && in_block) atomicMin(&bi.shrow[pos], t);
+  sm_bar_sync();
+  if (t < sd.slen) {
+    const bool ok = in_block && bi.shrow[pos] == t;
+    if (ok) bi.shpos[t] = pos;
+    else if (report && p.status) atomicOr(p.status, DARD_STATUS_BAD_SHADOW);
+  }
+  sm_bar_sync();
+  if (bi.shrow[t] == INT_MAX) bi.shrow[t] = -1;
+  sm_bar_sync();
+}
+
+__device__ __forceinline__ RowInfo row_info(const SeqDesc& sd, const BlockInfo& bi, int r) {
+  RowInfo q{0, kStateU, 0.f, -1, 1};
+  if (r < sd.n_orig) {
+    const int j = r - sd.b0;
+    if (j >= 0 && j < sd.blen) {
+      q.i = j;
+      q.si = bi.st[j];
+      q.ci = bi.cf[j];
+    } else {
+      q.si = (r < sd.b0) ? kStateU : kStateM;  // decoded context / future blocks
+    }
+  } else if (r < sd.n_orig + sd.slen) {
+    const int j = bi.shpos[r - sd.n_orig];
+    q.qs = 1;
+    if (j >= 0) {
+      q.i = j;
+      q.si = bi.st[j];
+      q.ci = bi.cf[j];
+    } else {
+      q.store = 0;
+    }
+  } else {
+    q.store = 0;
+  }
+  return q;
+}
+
+// Sec. 3.2: does query q take the shadow copy s^j (true) or x^j (false) of block position j?
+__device__ __forceinline__ bool takes_shadow(const RowInfo& q, int sj, float cj, int j) {
+  if (sj == kStateU) return q.qs && j == q.i;           // blocks 3/6: only the own position
+  if (sj == kStateM) return q.qs || q.si != kStateM;    // block 1 keeps x, all others s
+  if (q.si == kStateM) return q.qs;                     // block 1: x, block 4: s
+  if (q.si == kStateU) return true;                     // blocks 3/6: C keys from s
+  return !(q.ci <= cj) || (q.qs && j == q.i);           // blocks 2/5: Eq. 3
+}
+
+// Whether key row kr (sequence-relative) is attended by query q.
+__device__ __forceinline__ bool key_visible(const RowInfo& q, const BlockInfo& bi,
+                                            const SeqDesc& sd, int kr) {
+  if (kr >= sd.n_orig + sd.slen) return false;
+  if (kr >= sd.n_orig) {
+    const int j = bi.shpos[kr - sd.n_orig];
+    return j >= 0 && takes_shadow(q, bi.st[j], bi.cf[j], j);
+  }
+  const int j = kr - sd.b0;
+  if (j >= 0 && j < sd.blen) return !(bi.shrow[j] >= 0 && takes_shadow(q, bi.st[j], bi.cf[j], j));
+  return true;
+}
+
+__device__ __forceinline__ bool tile_needs_mask(const SeqDesc& sd, int kt0) {
+  return (kt0 + kBN > sd.n_orig) ||
+         (sd.blen > 0 && kt0 < sd.b0 + sd.blen && kt0 + kBN > sd.b0);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+struct __align__(8) TcCtl {
+  uint64_t q_full, k_full, k_empty, v_full, v_empty, s_full, p_full, pv_done;
+  uint32_t tmem_base;
+  int32_t abort;
+  BlockInfo bi;
+};
+
+template <int D>
+constexpr size_t tc_smem_bytes() {
+  return 1024 /*alignment slack*/ + 3 * static_cast<size_t>(kBM) * D * 2 + sizeof(TcCtl);
+}
+
+__device__ __forceinline__ void flag_timeout(const AttnParams& p, TcCtl& ctl) {
+  ctl.abort = 1;
+  if (p.status) atomicOr(p.status, DARD_STATUS_TIMEOUT);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, 2)
+    attn_tc(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmq,
+            const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv) {
+  constexpr int kSub = D / 64;                    // 128-byte (64 x bf16) column blocks
+  constexpr uint32_t kSubBytes = kBM * 128;       // one 128-row x 128-byte swizzled block
+  constexpr uint32_t kTileBytes = kSub * kSubBytes;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sQ = base;
+  uint8_t* sK = sQ + kTileBytes;
+  uint8_t* sV = sK + kTileBytes;
+  TcCtl& ctl = *reinterpret_cast<TcCtl*>(sV + kTileBytes);
+
+  int seq, qt, h;
+  decode_work(p, blockIdx.x, seq, qt, h);
+  const SeqDesc sd = p.seq[seq];
+  const int rows_seq = sd.n_orig + sd.slen;
+  const int n_kt = (rows_seq + kBN - 1) / kBN;
+  const int q0 = qt * kBM;
+  const int g = h / (p.hq / p.hkv);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&ctl.q_full, 1);
+    mbar_init(&ctl.k_full, 1);
+    mbar_init(&ctl.k_empty, 1);
+    mbar_init(&ctl.v_full, 1);
+    mbar_init(&ctl.v_empty, 1);
+    mbar_init(&ctl.s_full, 1);
+    mbar_init(&ctl.p_full, 4);
+    mbar_init(&ctl.pv_done, 1);
+    ctl.abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 4) {
+    tmem_alloc<kTmemCols>(&ctl.tmem_base);
+    tmem_relinquish();
+  }
+  if (warp < 4) load_block_info(p, sd, ctl.bi, qt == 0 && h == 0);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tS = ctl.tmem_base;
+  const uint32_t tO = ctl.tmem_base + 128;
+  volatile int32_t* abort_flag = &ctl.abort;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmq);
+      tma_prefetch_desc(&tmk);
+      tma_prefetch_desc(&tmv);
+      const int row0 = sd.row_base;
+      mbar_arrive_expect_tx(&ctl.q_full, kTileBytes);
+#pragma unroll
+      for (int s = 0; s < kSub; ++s)
+        tma_load_2d(sQ + s * kSubBytes, &tmq, &ctl.q_full, h * D + s * 64, row0 + q0);
+      int issued = 0;
+      for (int j = 0; j < n_kt && !*abort_flag; ++j) {
+        if (j > 0 && !mbar_wait(&ctl.k_empty, (j - 1) & 1)) { flag_timeout(p, ctl); break; }
+        mbar_arrive_expect_tx(&ctl.k_full, kTileBytes);
+#pragma unroll
+        for (int s = 0; s < kSub; ++s)
+          tma_load_2d(sK + s * kSubBytes, &tmk, &ctl.k_full, g * D + s * 64, row0 + j * kBN);
+        if (j > 0 && !mbar_wait(&ctl.v_empty, (j - 1) & 1)) { flag_timeout(p, ctl); issued = 2 * j + 1; break; }
+        mbar_arrive_expect_tx(&ctl.v_full, kTileBytes);
+#pragma unroll
+        for (int s = 0; s < kSub; ++s)
+          tma_load_2d(sV + s * kSubBytes, &tmv, &ctl.v_full, g * D + s * 64, row0 + j * kBN);
+        issued = 2 * j + 2;
+      }
+      if (*abort_flag && issued > 0) {
+        // let the copies already in flight land before the CTA's shared memory is released
+        const int jk = (issued - 1) / 2;
+        mbar_wait(&ctl.k_full, jk & 1);
+        if ((issued & 1) == 0) mbar_wait(&ctl.v_full, jk & 1);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kBN, 0, 0);
+      constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
+      const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK), av = smem_u32(sV);
+      bool ok = mbar_wait(&ctl.q_full, 0);
+      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
+        ok = mbar_wait(&ctl.k_full, j & 1);
+        if (ok && j > 0) ok = mbar_wait(&ctl.pv_done, (j - 1) & 1);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (ks >> 2) * kSubBytes + (ks & 3) * 32;
+          mma_ss(tS, smem_desc_sw128(aq + off, 16, 1024), smem_desc_sw128(ak + off, 16, 1024),
+                 kIdS, ks > 0);
+        }
+        mma_commit(&ctl.s_full);
+        mma_commit(&ctl.k_empty);
+        ok = mbar_wait(&ctl.p_full, j & 1);
+        if (ok) ok = mbar_wait(&ctl.v_full, j & 1);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int ks = 0; ks < kBN / 16; ++ks)
+          mma_ts(tO, tS + ks * 8, smem_desc_sw128(av + ks * 2048, kSubBytes, 1024), kIdO,
+                 (j > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&ctl.pv_done);
+        mma_commit(&ctl.v_empty);
+      }
+      if (!ok) flag_timeout(p, ctl);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax + epilogue
+    const int t = threadIdx.x;
+    const RowInfo q = row_info(sd, ctl.bi, q0 + t);
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const float sl = p.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_kt; ++j) {
+      const int kt0 = j * kBN;
+      uint32_t vis[4] = {~0u, ~0u, ~0u, ~0u};
+      const bool masked = tile_needs_mask(sd, kt0);
+      if (masked) {
+        for (int k = 0; k < kBN; ++k)
+          if (!key_visible(q, ctl.bi, sd, kt0 + k)) vis[k >> 5] &= ~(1u << (k & 31));
+      }
+      ok = !*abort_flag && mbar_wait(&ctl.s_full, j & 1);
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      tc_fence_after();
+      float s[kBN];
+#pragma unroll
+      for (int c = 0; c < kBN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tS + lane_off + c * 32, r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(r[e]);
+      }
+      float mt = -INFINITY;
+      if (masked) {
+#pragma unroll
+        for (int k = 0; k < kBN; ++k) {
+          s[k] = ((vis[k >> 5] >> (k & 31)) & 1u) ? s[k] : -INFINITY;
+          mt = fmaxf(mt, s[k]);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < kBN; ++k) mt = fmaxf(mt, s[k]);
+      }
+      // Raise the reference maximum on the first finite value, or when the tile maximum
+      // exceeds it by more than 2^kRescaleLog2 in probability; O is rescaled only then.
+      float m_new = m_run;
+      if (m_run == -INFINITY) m_new = mt;
+      else if ((mt - m_run) * sl > kRescaleLog2) m_new = mt;
+      const bool rescale = (m_new != m_run) && (m_run != -INFINITY);
+      const float alpha = rescale ? ex2_approx((m_run - m_new) * sl) : 1.f;
+      if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tO + lane_off + c * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+          tmem_st32(tO + lane_off + c * 32, r);
+        }
+      }
+      l_run *= alpha;
+      m_run = m_new;
+      const float mL = (m_run == -INFINITY) ? 0.f : m_run * sl;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const float a = ex2_approx(fmaf(s[half * 64 + 2 * e], sl, -mL));
+          const float b = ex2_approx(fmaf(s[half * 64 + 2 * e + 1], sl, -mL));
+          l_run += a + b;
+          pk[e] = pack_bf16x2(a, b);
+        }
+        tmem_st32(tS + lane_off + half * 32, pk);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.p_full);
+    }
+    if (ok) ok = mbar_wait(&ctl.pv_done, (n_kt - 1) & 1);
+    if (!__all_sync(0xffffffffu, ok)) {
+      if (lane == 0) flag_timeout(p, ctl);
+    } else {
+      tc_fence_after();
+      const int r = q0 + t;
+      const bool store = q.store && r < rows_seq;
+      const float inv_l = 1.0f / l_run;
+      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o) +
+                           (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t rr[32];
+        tmem_ld32(tO + lane_off + c * 32, rr);
+        tmem_wait_ld();
+        if (store) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e)
+            pk[e] = pack_bf16x2(__uint_as_float(rr[2 * e]) * inv_l,
+                                __uint_as_float(rr[2 * e + 1]) * inv_l);
+          uint4* dst = reinterpret_cast<uint4*>(out + c * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    tc_fence_after();
+    tmem_dealloc<kTmemCols>(ctl.tmem_base);
+  }
+}
+
+// ---------------------------------------------------------------- fp32 CUDA-core path
+template <int D>
+__global__ void __launch_bounds__(128) attn_simt(const __grid_constant__ AttnParams p) {
+  constexpr int kPer = D / 32;
+  __shared__ BlockInfo bi;
+  int seq, qt, h;
+  decode_work(p, blockIdx.x, seq, qt, h);
+  const SeqDesc sd = p.seq[seq];
+  const int rows_seq = sd.n_orig + sd.slen;
+  const int g = h / (p.hq / p.hkv);
+  load_block_info(p, sd, bi, qt == 0 && h == 0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* Q = static_cast<const float*>(p.q);
+  const float* K = static_cast<const float*>(p.k);
+  const float* V = static_cast<const float*>(p.v);
+  float* O = static_cast<float*>(p.o);
+  const float scale = p.scale;
+  for (int rr = 0; rr < 32; ++rr) {
+    const int r = qt * kBM + warp * 32 + rr;
+    if (r >= rows_seq) break;
+    const RowInfo q = row_info(sd, bi, r);
+    if (!q.store) continue;
+    const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D;
+    float qv[kPer], acc[kPer];
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      qv[e] = Q[qoff + lane + 32 * e];
+      acc[e] = 0.f;
+    }
+    float m = -INFINITY, l = 0.f;
+    for (int kr = 0; kr < rows_seq; ++kr) {
+      if (!key_visible(q, bi, sd, kr)) continue;
+      const size_t koff = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D;
+      float dot = 0.f;
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) dot = fmaf(qv[e], K[koff + lane + 32 * e], dot);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+      const float z = dot * scale;
+      const float m_new = fmaxf(m, z);
+      const float alpha = (m == -INFINITY) ? 0.f : expf(m - m_new);
+      const float pz = expf(z - m_new);
+      l = l * alpha + pz;
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) acc[e] = fmaf(pz, V[koff + lane + 32 * e], acc[e] * alpha);
+      m = m_new;
+    }
+    const float inv_l = 1.0f / l;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) O[qoff + lane + 32 * e] = acc[e] * inv_l;
+  }
+}
+
+// ---------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+bool make_map(CUtensorMap* m, const void* ptr, int heads, int d, int rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(heads) * d, static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(heads) * d * 2};
+  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kBM)};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// cudaFuncSetAttribute once per (kernel, device).
+template <class F>
+cudaError_t ensure_smem_attr(F* kernel, size_t bytes, std::atomic<uint64_t>& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (done.load(std::memory_order_acquire) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(bytes));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
+}
+
+template <int D>
+cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
+  static std::atomic<uint64_t> attr_done{0};
+  CUtensorMap mq, mk, mv;
+  if (!make_map(&mq, p.q, p.hq, D, p.total_rows) || !make_map(&mk, p.k, p.hkv, D, p.total_rows) ||
+      !make_map(&mv, p.v, p.hkv, D, p.total_rows))
+    return cudaErrorInvalidValue;
+  const size_t smem = tc_smem_bytes<D>();
+  cudaError_t e = ensure_smem_attr(attn_tc<D>, smem, attr_done);
+  if (e != cudaSuccess) return e;
+  attn_tc<D><<<p.total_work, kTcThreads, smem, stream>>>(p, mq, mk, mv);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
+                             char* err, size_t err_len) {
+  cudaError_t e;
+  if (a.dtype == DARD_F32) {
+    if (a.head_dim == 64) attn_simt<64><<<p.total_work, 128, 0, stream>>>(p);
+    else attn_simt<128><<<p.total_work, 128, 0, stream>>>(p);
+    e = cudaGetLastError();
+  } else {
+    e = a.head_dim == 64 ? launch_tc<64>(p, stream) : launch_tc<128>(p, stream);
+  }
+  if (e != cudaSuccess) {
+    snprintf(err, err_len, "attention launch failed: %s", cudaGetErrorString(e));
+    return DARD_ERR_CUDA;
+  }
+  return DARD_OK;
+}
+
+}  // namespace dard

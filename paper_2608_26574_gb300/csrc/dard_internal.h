@@ -1,0 +1,79 @@
+// dard_internal.h - launch parameter blocks shared by the C-ABI layer and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <cstddef>
+#include <cstdint>
+
+#include "dard.h"
+
+namespace dard {
+
+constexpr int kStateM = 0, kStateC = 1, kStateU = 2;
+
+// ------------------------------------------------------------------ attention
+// Per-sequence layout, copied by value into the kernel parameters (no device metadata).
+struct SeqDesc {
+  int32_t row_base;   // first row of the sequence in Q/K/V/O
+  int32_t n_orig;     // N
+  int32_t b0;         // block start
+  int32_t blen;       // B
+  int32_t slen;       // S
+  int32_t blk_off;    // offset of the block in state / prev_conf
+  int32_t sh_off;     // offset of the shadow rows in shadow_src
+  int32_t n_qtiles;   // ceil((N + S) / 128)
+};
+
+struct AttnParams {
+  const uint8_t* state;
+  const float* prev_conf;
+  const int32_t* shadow_src;
+  void* o;
+  const void* q;
+  const void* k;
+  const void* v;
+  uint32_t* status;
+  float scale;               // softmax scale
+  float scale_log2;          // scale * log2(e)
+  int32_t hq, hkv, head_dim, num_seqs;
+  int32_t total_rows;
+  int32_t total_work;        // number of (sequence, q-tile, head) work items
+  // Work items in longest-first order: sequence order[r] owns items
+  // [work_prefix[r], work_prefix[r+1]), laid out q-tile major, head minor.
+  int32_t order[DARD_MAX_SEQS];
+  int32_t work_prefix[DARD_MAX_SEQS + 1];
+  SeqDesc seq[DARD_MAX_SEQS];
+};
+
+dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
+                             char* err, size_t err_len);
+
+// ------------------------------------------------------------------ scoring
+struct ScoreParams {
+  const void* lx;
+  const void* ls;
+  const uint8_t* state_in;
+  float* conf;
+  int32_t* token;
+  uint8_t* state_out;
+  float* w_out;
+  int32_t* counts;
+  uint32_t* status;
+  // workspace
+  float4* partial;     // [rows * nsplit] (max, sum, argmax bits, unused)
+  uint32_t* row_ctr;   // [rows]
+  uint32_t* seq_ctr;   // [num_seqs]
+  uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 0 otherwise
+  int64_t row_stride;
+  int32_t vocab, rows, num_seqs, nsplit, chunk;
+  float tau_c, tau_u, lambda, p0;
+  int32_t blk_off[DARD_MAX_SEQS + 1];
+};
+
+constexpr int kScoreThreads = 256;
+constexpr int kScoreMaxSplit = 64;
+
+size_t score_workspace_bytes(int32_t rows, int32_t num_seqs);
+dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
+                         char* err, size_t err_len);
+
+}  // namespace dard

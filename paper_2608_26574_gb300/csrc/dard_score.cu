@@ -1,0 +1,456 @@
+// dard_score.cu - confidence scoring and state transition of one DARD step (sm_103a).
+//
+// Implements Eq. 1 (max-probability and argmax), Eq. 5-6 (verification-outcome kernel and
+// guidance weight), Eq. 7 (logit mixing) and Eq. 8 (three-state transition) in the order of
+// Algorithm 1 of arXiv 2608.26574:
+//
+//   pass 1  rows in state C or U read their shadow logits once and are decided; C rows
+//           record whether they were promoted (P) or demoted (D);
+//   pass 2  rows in state M read both logit rows once, weight them by w from P and D of
+//           their own block and are decided.
+//
+// Both passes split every vocabulary row over `nsplit` CTAs (256 threads, 128-bit streaming
+// loads, warp-shuffle merge of (max, sum of exp, argmax)); the last CTA of a row, found with
+// an atomic counter, merges the per-split partials in a fixed order and writes the row's
+// outputs. Pass 2 is launched as a programmatic dependent of pass 1: its CTAs load their
+// logits while pass 1 finishes and only then wait for pass 1's results.
+#include <cfloat>
+#include <climits>
+#include <cstdio>
+
+#include "dard_internal.h"
+#include "dard_ptx.cuh"
+
+namespace dard {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kWarps = kScoreThreads / 32;
+
+struct Acc {
+  float m;   // running maximum
+  float s;   // sum of exp(x - m)
+  int idx;   // lowest index attaining m
+};
+
+// Merge of two partial softmax summaries; equal maxima keep the lower index.
+__device__ __forceinline__ Acc acc_merge(const Acc& a, const Acc& b) {
+  const bool b_wins = (b.m > a.m) || (b.m == a.m && b.idx < a.idx);
+  const Acc hi = b_wins ? b : a;
+  const Acc lo = b_wins ? a : b;
+  const float f = (lo.m == -INFINITY) ? 0.f : ex2_approx((lo.m - hi.m) * kLog2e);
+  return {hi.m, fmaf(lo.s, f, hi.s), hi.idx};
+}
+
+__device__ __forceinline__ Acc warp_merge(Acc a) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    Acc b;
+    b.m = __shfl_xor_sync(0xffffffffu, a.m, off);
+    b.s = __shfl_xor_sync(0xffffffffu, a.s, off);
+    b.idx = __shfl_xor_sync(0xffffffffu, a.idx, off);
+    a = acc_merge(a, b);
+  }
+  return a;
+}
+
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+// Element access for the two logit types; W elements per 16-byte vector.
+struct Bf16 {
+  static constexpr int W = 8;
+  static constexpr int kBytes = 2;
+  __device__ static float get(const uint4& v, int e) {
+    const uint32_t w = (e >> 1) == 0 ? v.x : (e >> 1) == 1 ? v.y : (e >> 1) == 2 ? v.z : v.w;
+    return __uint_as_float((e & 1) ? (w & 0xffff0000u) : (w << 16));
+  }
+  __device__ static float scalar(const char* p) {
+    return __uint_as_float(static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(p)) << 16);
+  }
+};
+struct F32 {
+  static constexpr int W = 4;
+  static constexpr int kBytes = 4;
+  __device__ static float get(const uint4& v, int e) {
+    const uint32_t w = e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+    return __uint_as_float(w);
+  }
+  __device__ static float scalar(const char* p) { return *reinterpret_cast<const float*>(p); }
+};
+
+constexpr uint32_t kNegInfBits = 0xff800000u;
+
+// Loads vector v of this thread's round starting at element `base`; elements at or past c1
+// read as -inf (neutral for max, argmax and the exp-sum).
+template <class T>
+__device__ __forceinline__ uint4 load_vec(const char* row, int e0, int c1) {
+  if (e0 + T::W <= c1) return ld_stream(row + static_cast<size_t>(e0) * T::kBytes);
+  uint4 r;
+  uint32_t* w = &r.x;
+  if (T::kBytes == 4) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      w[e] = (e0 + e < c1) ? __float_as_uint(T::scalar(row + static_cast<size_t>(e0 + e) * 4))
+                           : kNegInfBits;
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int a = e0 + 2 * k, b = a + 1;
+      const uint32_t lo = a < c1 ? *reinterpret_cast<const uint16_t*>(row + static_cast<size_t>(a) * 2)
+                                 : (kNegInfBits >> 16);
+      const uint32_t hi = b < c1 ? *reinterpret_cast<const uint16_t*>(row + static_cast<size_t>(b) * 2)
+                                 : (kNegInfBits >> 16);
+      w[k] = lo | (hi << 16);
+    }
+  }
+  return r;
+}
+
+// Folds VPT*W values (given by `val(v, e)`, element index `base + (v*256 + tid)*W + e`) into
+// the running accumulator: max/argmax first, then the exp-sum against the updated maximum.
+template <class T, int VPT, class ValFn>
+__device__ __forceinline__ void fold_round(Acc& acc, int base, ValFn val) {
+  float m = -INFINITY;
+  int idx = INT_MAX;
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+#pragma unroll
+    for (int e = 0; e < T::W; ++e) {
+      const float x = val(v, e);
+      if (x > m) {
+        m = x;
+        idx = base + (v * kScoreThreads + static_cast<int>(threadIdx.x)) * T::W + e;
+      }
+    }
+  }
+  if (m > acc.m) {
+    acc.s = (acc.m == -INFINITY) ? 0.f : acc.s * ex2_approx((acc.m - m) * kLog2e);
+    acc.m = m;
+    acc.idx = idx;
+  }
+  const float mL = (acc.m == -INFINITY) ? 0.f : acc.m * kLog2e;
+  float s = 0.f;
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+#pragma unroll
+    for (int e = 0; e < T::W; ++e) s += ex2_approx(fmaf(val(v, e), kLog2e, -mL));
+  }
+  acc.s += s;
+}
+
+__device__ __forceinline__ Acc block_merge(Acc a, Acc* smem) {
+  a = warp_merge(a);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) smem[warp] = a;
+  __syncthreads();
+  if (warp == 0) {
+    a = lane < kWarps ? smem[lane] : Acc{-INFINITY, 0.f, INT_MAX};
+    a = warp_merge(a);
+  }
+  return a;  // valid in warp 0
+}
+
+__device__ __forceinline__ int seq_of_row(const ScoreParams& p, int row) {
+  int lo = 0, hi = p.num_seqs;  // blk_off[lo] <= row < blk_off[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (p.blk_off[mid] <= row) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ int load_state(const ScoreParams& p, int row, bool report) {
+  int s = p.state_in[row];
+  if (s > 2) {
+    if (report && p.status) atomicOr(p.status, DARD_STATUS_BAD_STATE);
+    s = kStateM;
+  }
+  return s;
+}
+
+// Publishes this CTA's partial; returns true (in every thread) for the row's last CTA.
+__device__ __forceinline__ bool publish_partial(const ScoreParams& p, int row, int split,
+                                                const Acc& a, int* s_flag) {
+  if (threadIdx.x == 0) {
+    p.partial[static_cast<size_t>(row) * p.nsplit + split] =
+        make_float4(a.m, a.s, __int_as_float(a.idx), 0.f);
+    __threadfence();
+    const uint32_t prev = atomicAdd(&p.row_ctr[row], 1u);
+    *s_flag = (prev == static_cast<uint32_t>(p.nsplit - 1));
+  }
+  __syncthreads();
+  return *s_flag != 0;
+}
+
+// Merges the row's partials in split order (warp 0); returns the row summary in lane 0.
+__device__ __forceinline__ Acc merge_partials(const ScoreParams& p, int row) {
+  __threadfence();
+  Acc a{-INFINITY, 0.f, INT_MAX};
+  const int lane = threadIdx.x & 31;
+  for (int k = lane; k < p.nsplit; k += 32) {
+    const float4 v = __ldcg(&p.partial[static_cast<size_t>(row) * p.nsplit + k]);
+    a = acc_merge(a, Acc{v.x, v.y, __float_as_int(v.z)});
+  }
+  return warp_merge(a);
+}
+
+// Eq. 1 and Eq. 8 on a merged row; writes conf / token / state and returns the new state.
+__device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const Acc& a,
+                                            float w) {
+  const float z = a.s;
+  const bool valid = isfinite(z) && z > 0.f;
+  const float c = valid ? 1.0f / z : 0.f;
+  const int ns = !valid ? kStateM : (c <= p.tau_c ? kStateM : (c <= p.tau_u ? kStateC : kStateU));
+  p.conf[row] = c;
+  p.token[row] = valid ? a.idx : -1;
+  p.state_out[row] = static_cast<uint8_t>(ns);
+  if (p.w_out) p.w_out[row] = w;
+  if (!valid && p.status) atomicOr(p.status, DARD_STATUS_INVALID_ROW);
+  p.row_ctr[row] = 0u;  // leave the workspace zeroed for the next call
+  return ns;
+}
+
+// One arrival per row of a sequence in pass 2; the last one writes the M/C/U counts.
+__device__ __forceinline__ void arrive_counts(const ScoreParams& p, int seq) {
+  // called by a whole warp
+  const int lane = threadIdx.x & 31;
+  uint32_t last = 0;
+  const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
+  if (lane == 0) {
+    __threadfence();
+    last = atomicAdd(&p.seq_ctr[seq], 1u) == static_cast<uint32_t>(blen - 1);
+  }
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
+  __threadfence();
+  int cnt[3] = {0, 0, 0};
+  for (int j = lane; j < blen; j += 32) {
+    const int s = __ldcg(p.state_out + b0 + j);
+    cnt[0] += s == kStateM;
+    cnt[1] += s == kStateC;
+    cnt[2] += s == kStateU;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+    for (int k = 0; k < 3; ++k) cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], off);
+  if (lane == 0) {
+    p.counts[seq * 3 + 0] = cnt[0];
+    p.counts[seq * 3 + 1] = cnt[1];
+    p.counts[seq * 3 + 2] = cnt[2];
+    p.seq_ctr[seq] = 0u;
+  }
+}
+
+template <class T, int VPT>
+__global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_constant__ ScoreParams p) {
+  grid_dep_launch();  // pass 2 may start loading its logits right away
+  __shared__ Acc s_acc[kWarps];
+  __shared__ int s_last;
+  const int row = blockIdx.y, split = blockIdx.x;
+  const int st = load_state(p, row, split == 0);
+  if (st == kStateM) {
+    if (split == 0) p.pd_flag[row] = 0;
+    return;
+  }
+  const char* rowp = static_cast<const char*>(p.ls) + static_cast<size_t>(row) * p.row_stride * T::kBytes;
+  const int c0 = split * p.chunk;
+  const int c1 = min(p.vocab, c0 + p.chunk);
+  Acc acc{-INFINITY, 0.f, INT_MAX};
+  for (int base = c0; base < c1; base += kScoreThreads * VPT * T::W) {
+    uint4 r[VPT];
+#pragma unroll
+    for (int v = 0; v < VPT; ++v)
+      r[v] = load_vec<T>(rowp, base + (v * kScoreThreads + threadIdx.x) * T::W, c1);
+    fold_round<T, VPT>(acc, base, [&](int v, int e) { return T::get(r[v], e); });
+  }
+  acc = block_merge(acc, s_acc);
+  if (!publish_partial(p, row, split, acc, &s_last)) return;
+  if (threadIdx.x >= 32) return;
+  const Acc a = merge_partials(p, row);
+  if (threadIdx.x == 0) {
+    const int ns = finalize_row(p, row, a, __int_as_float(0x7fc00000));
+    p.pd_flag[row] = (st == kStateC) ? (ns == kStateU ? 1 : (ns == kStateM ? 2 : 0)) : 0;
+  }
+}
+
+template <class T, int VPT>
+__global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_constant__ ScoreParams p) {
+  __shared__ Acc s_acc[kWarps];
+  __shared__ double s_red[2][kWarps];
+  __shared__ int s_last;
+  const int row = blockIdx.y, split = blockIdx.x;
+  const int st = load_state(p, row, false);
+  const int seq = seq_of_row(p, row);
+  if (st != kStateM) {
+    if (split == 0 && p.counts != nullptr && threadIdx.x < 32) {
+      grid_dep_wait();
+      arrive_counts(p, seq);
+    }
+    return;
+  }
+  const size_t roff = static_cast<size_t>(row) * p.row_stride * T::kBytes;
+  const char* xp = static_cast<const char*>(p.lx) + roff;
+  const char* sp = static_cast<const char*>(p.ls) + roff;
+  const int c0 = split * p.chunk;
+  const int c1 = min(p.vocab, c0 + p.chunk);
+
+  // The first round's loads do not depend on pass 1: issue them before waiting for it.
+  uint4 rx[VPT], rs[VPT];
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+    const int e0 = c0 + (v * kScoreThreads + threadIdx.x) * T::W;
+    rx[v] = load_vec<T>(xp, e0, c1);
+    rs[v] = load_vec<T>(sp, e0, c1);
+  }
+  grid_dep_wait();
+
+  // Eq. 5-6: w from the verification outcomes of this block (fp64, tree-summed).
+  const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
+  const int i = row - b0;
+  double pp = 0.0, dd = 0.0;
+  for (int j = threadIdx.x; j < blen; j += kScoreThreads) {
+    const int f = __ldcg(p.pd_flag + b0 + j);
+    if (f != 0) {
+      const double kij = pow(static_cast<double>(p.lambda), static_cast<double>(abs(i - j)));
+      if (f == 1) pp += kij; else dd += kij;
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    pp += __shfl_xor_sync(0xffffffffu, pp, off);
+    dd += __shfl_xor_sync(0xffffffffu, dd, off);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    s_red[0][threadIdx.x >> 5] = pp;
+    s_red[1][threadIdx.x >> 5] = dd;
+  }
+  __syncthreads();
+  pp = 0.0;
+  dd = 0.0;
+#pragma unroll
+  for (int k = 0; k < kWarps; ++k) {
+    pp += s_red[0][k];
+    dd += s_red[1][k];
+  }
+  const double p0 = static_cast<double>(p.p0);
+  const float w = static_cast<float>((pp + p0) / (pp + dd + p0));
+
+  // Eq. 7 in fp32, one rounding per operation: mix = ls + w * (lx - ls).
+  auto mix = [&](const uint4& vx, const uint4& vs, int e) {
+    const float lx = T::get(vx, e), ls = T::get(vs, e);
+    return __fadd_rn(ls, __fmul_rn(w, __fsub_rn(lx, ls)));
+  };
+  Acc acc{-INFINITY, 0.f, INT_MAX};
+  fold_round<T, VPT>(acc, c0, [&](int v, int e) { return mix(rx[v], rs[v], e); });
+  for (int base = c0 + kScoreThreads * VPT * T::W; base < c1; base += kScoreThreads * VPT * T::W) {
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int e0 = base + (v * kScoreThreads + threadIdx.x) * T::W;
+      rx[v] = load_vec<T>(xp, e0, c1);
+      rs[v] = load_vec<T>(sp, e0, c1);
+    }
+    fold_round<T, VPT>(acc, base, [&](int v, int e) { return mix(rx[v], rs[v], e); });
+  }
+  acc = block_merge(acc, s_acc);
+  if (!publish_partial(p, row, split, acc, &s_last)) return;
+  if (threadIdx.x >= 32) return;
+  const Acc a = merge_partials(p, row);
+  if (threadIdx.x == 0) finalize_row(p, row, a, w);
+  if (p.counts != nullptr) {
+    __syncwarp();
+    arrive_counts(p, seq);
+  }
+}
+
+// Zeroes the counts of sequences without block rows (they get no arrivals).
+__global__ void zero_empty_counts(const __grid_constant__ ScoreParams p) {
+  for (int s = threadIdx.x; s < p.num_seqs; s += blockDim.x)
+    if (p.blk_off[s + 1] == p.blk_off[s]) {
+      p.counts[s * 3 + 0] = 0;
+      p.counts[s * 3 + 1] = 0;
+      p.counts[s * 3 + 2] = 0;
+    }
+}
+
+template <class T, int VPT>
+cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
+  dim3 grid(p.nsplit, p.rows);
+  score_pass1<T, VPT><<<grid, kScoreThreads, 0, stream>>>(p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kScoreThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, score_pass2<T, VPT>, p);
+}
+
+}  // namespace
+
+size_t score_workspace_bytes(int32_t rows, int32_t num_seqs) {
+  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+  return up(static_cast<size_t>(rows) * kScoreMaxSplit * sizeof(float4)) +
+         up(static_cast<size_t>(rows) * sizeof(uint32_t)) +
+         up(static_cast<size_t>(num_seqs) * sizeof(uint32_t)) + up(static_cast<size_t>(rows));
+}
+
+dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
+                         char* err, size_t err_len) {
+  const bool bf16 = a.dtype == DARD_BF16;
+  const int W = bf16 ? 8 : 4;
+  // Vectors per thread per round: 4, or 2 when the grid would otherwise leave SMs idle.
+  int vpt = 4;
+  int per_round = kScoreThreads * vpt * W;
+  if (static_cast<long long>(p.rows) * ((p.vocab + per_round - 1) / per_round) < 1216) vpt = 2;
+  per_round = kScoreThreads * vpt * W;
+  int nsplit = (p.vocab + per_round - 1) / per_round;
+  int rounds = 1;
+  if (nsplit > kScoreMaxSplit) {
+    rounds = (nsplit + kScoreMaxSplit - 1) / kScoreMaxSplit;
+    nsplit = (p.vocab + per_round * rounds - 1) / (per_round * rounds);
+  }
+  p.nsplit = nsplit;
+  p.chunk = per_round * rounds;
+
+  char* ws = static_cast<char*>(a.workspace);
+  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+  p.partial = reinterpret_cast<float4*>(ws);
+  ws += up(static_cast<size_t>(p.rows) * kScoreMaxSplit * sizeof(float4));
+  p.row_ctr = reinterpret_cast<uint32_t*>(ws);
+  ws += up(static_cast<size_t>(p.rows) * sizeof(uint32_t));
+  p.seq_ctr = reinterpret_cast<uint32_t*>(ws);
+  ws += up(static_cast<size_t>(p.num_seqs) * sizeof(uint32_t));
+  p.pd_flag = reinterpret_cast<uint8_t*>(ws);
+
+  cudaError_t e = cudaSuccess;
+  bool any_empty = false;
+  for (int s = 0; s < p.num_seqs; ++s) any_empty |= p.blk_off[s + 1] == p.blk_off[s];
+  if (p.counts != nullptr && any_empty) {
+    zero_empty_counts<<<1, 256, 0, stream>>>(p);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess && p.rows > 0) {
+    if (bf16) e = vpt == 4 ? launch_pair<Bf16, 4>(p, stream) : launch_pair<Bf16, 2>(p, stream);
+    else e = vpt == 4 ? launch_pair<F32, 4>(p, stream) : launch_pair<F32, 2>(p, stream);
+  }
+  if (e != cudaSuccess) {
+    snprintf(err, err_len, "scoring launch failed: %s", cudaGetErrorString(e));
+    return DARD_ERR_CUDA;
+  }
+  return DARD_OK;
+}
+
+}  // namespace dard

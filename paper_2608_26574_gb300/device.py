@@ -1,0 +1,72 @@
+"""Device-side holder of one DARD step's inputs and outputs (torch for memory only).
+
+``DeviceStep`` uploads a seeded ``workloads.Workload`` (one layer, or all layers) to the GPU,
+owns the output tensors and the scoring workspace, and calls the two C-ABI entry points
+through ``binding``. It is what the tests, ``bench.py`` and ``smoke()`` drive.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import binding as B
+from .workloads import Workload
+
+
+def to_device(a: np.ndarray, dtype: str, device) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if dtype == "bf16":
+        t = t.to(torch.bfloat16)  # values are already bf16-exact: the conversion is exact
+    return t.to(device)
+
+
+class DeviceStep:
+    def __init__(self, wl: Workload, device="cuda", layers=None, attention=True, scoring=True):
+        self.wl = wl
+        self.device = torch.device(device)
+        dt = wl.dtype
+        self.n_orig = np.array([s.n_orig for s in wl.seqs], dtype=np.int32)
+        self.block_start = np.array([s.block_start for s in wl.seqs], dtype=np.int32)
+        self.block_len = np.array([s.block_len for s in wl.seqs], dtype=np.int32)
+        self.shadow_len = np.array([s.n_shadow for s in wl.seqs], dtype=np.int32)
+        dev = self.device
+        self.state = torch.from_numpy(wl.state_all()).to(dev)
+        self.prev_conf = torch.from_numpy(wl.prev_conf_all()).to(dev)
+        sh = wl.shadow_src_all()
+        self.shadow_src = torch.from_numpy(sh if len(sh) else np.zeros(1, np.int32)).to(dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.layers = []
+        if attention:
+            idx = range(len(wl.q)) if layers is None else layers
+            for li in idx:
+                q = to_device(wl.q[li], dt, dev)
+                k = to_device(wl.k[li], dt, dev)
+                v = to_device(wl.v[li], dt, dev)
+                self.layers.append((q, k, v, torch.empty_like(q)))
+        self.rows = wl.total_block
+        if scoring and wl.logits_s is not None:
+            self.lx = to_device(wl.logits_x, dt, dev)
+            self.ls = to_device(wl.logits_s, dt, dev)
+            nbytes = B.dard_score_workspace_size(self.rows, wl.vocab, len(wl.seqs))
+            self.workspace = torch.zeros(max(nbytes, 16), dtype=torch.uint8, device=dev)
+            r = max(self.rows, 1)
+            self.conf = torch.empty(r, dtype=torch.float32, device=dev)
+            self.token = torch.empty(r, dtype=torch.int32, device=dev)
+            self.state_out = torch.empty(r, dtype=torch.uint8, device=dev)
+            self.w_out = torch.empty(r, dtype=torch.float32, device=dev)
+            self.counts = torch.empty(3 * len(wl.seqs), dtype=torch.int32, device=dev)
+
+    def attention(self, layer: int = 0, scale: float = 0.0, stream=None, out=None):
+        q, k, v, o = self.layers[layer]
+        B.dard_step_attention(q, k, v, o if out is None else out, self.n_orig, self.block_start,
+                              self.block_len, self.shadow_len, self.state, self.prev_conf,
+                              self.shadow_src, scale=scale, status=self.status, stream=stream)
+        return o if out is None else out
+
+    def score(self, stream=None, w_out=True, counts=True, state_in=None):
+        wl = self.wl
+        B.dard_score_and_transition(
+            self.lx, self.ls, self.block_len, self.state if state_in is None else state_in,
+            wl.tau_c, wl.tau_u, wl.lam, wl.p0, self.conf, self.token, self.state_out,
+            self.workspace, w_out=self.w_out if w_out else None,
+            counts=self.counts if counts else None, status=self.status, stream=stream)

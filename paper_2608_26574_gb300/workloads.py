@@ -267,3 +267,53 @@ def scoring_bytes(wl: Workload) -> float:
     esz = 2 if wl.dtype == "bf16" else 4
     n_m = sum(int((s.state == STATE_M).sum()) for s in wl.seqs)
     return float(wl.vocab * esz * (wl.total_block + n_m))
+
+
+def custom(specs, hq: int, hkv: int, head_dim: int, dtype: str = "bf16", vocab: int = 0,
+           seed: int = 0, qkv_std: float | None = None, probe: bool = False,
+           logits: str = "spanning", logit_std: float = 3.0, tau=(0.5, 0.8)) -> Workload:
+    """A seeded workload from explicit per-sequence specs (edge cases, small shapes).
+
+    specs: list of dicts with n_orig, block_start, and either state (uint8 array) or
+    fractions (M, C, U) with block_len; optional prev_conf (float32 array) and shadow
+    ("paper", "candidates" or an explicit int array of original positions).
+    probe=True draws Q = 0 (uniform attention over the attended keys) and K, V ~ N(0, 1), so
+    that every attended key shows in the output with weight 1/N.
+    """
+    rng = np.random.default_rng(np.random.PCG64(seed))
+    tau_c, tau_u = tau
+    seqs = []
+    for sp in specs:
+        if "state" in sp:
+            st = np.asarray(sp["state"], dtype=np.uint8)
+            cf = np.empty(len(st), np.float32)
+            for code, lo, hi in ((STATE_M, 0.0, tau_c), (STATE_C, tau_c, tau_u), (STATE_U, tau_u, 1.0)):
+                sel = st == code
+                cf[sel] = lo + (hi - lo) * (1.0 - rng.random(int(sel.sum())))
+        else:
+            st, cf = _draw_states(rng, sp["block_len"], sp["fractions"], tau_c, tau_u)
+        if sp.get("prev_conf") is not None:
+            cf = np.asarray(sp["prev_conf"], dtype=np.float32)
+        shadow = sp.get("shadow", "paper")
+        src = _shadow(st, sp["block_start"], shadow) if isinstance(shadow, str) else \
+            np.asarray(shadow, dtype=np.int32)
+        seqs.append(Seq(sp["n_orig"], sp["block_start"], st, cf, src))
+    wl = Workload("custom", dtype, hq, hkv, head_dim, vocab, seqs, tau_c, tau_u)
+    std = (1.0 / math.sqrt(head_dim)) if qkv_std is None else qkv_std
+    rows = wl.total_rows
+    if probe:
+        q = np.zeros((rows, hq, head_dim), np.float32)
+        k = rng.standard_normal((rows, hkv, head_dim), dtype=np.float32)
+        v = rng.standard_normal((rows, hkv, head_dim), dtype=np.float32)
+    else:
+        q = rng.standard_normal((rows, hq, head_dim), dtype=np.float32) * np.float32(std)
+        k = rng.standard_normal((rows, hkv, head_dim), dtype=np.float32) * np.float32(std)
+        v = rng.standard_normal((rows, hkv, head_dim), dtype=np.float32) * np.float32(std)
+    if dtype == "bf16":
+        q, k, v = round_bf16(q), round_bf16(k), round_bf16(v)
+    wl.q, wl.k, wl.v = [q], [k], [v]
+    if vocab > 0:
+        nrows = wl.total_block
+        wl.logits_x = _logits(rng, nrows, vocab, logit_std, dtype, logits, 0.5, 6.0)
+        wl.logits_s = _logits(rng, nrows, vocab, logit_std, dtype, logits, 0.5, 6.0)
+    return wl

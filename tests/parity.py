@@ -1,0 +1,109 @@
+"""Comparison of the CUDA path's outputs with the CPU oracle on the same seeded inputs."""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle as orc
+
+BORDER = 1e-5      # |c - tau| below this: the transition may legitimately go either way
+NEAR_TIE = 1e-3    # top-2 logit gap below this: the argmax may legitimately differ
+CONF_TOL = 1e-4    # confidences, fp32 accumulation
+ATT_MAX_ABS = 2e-2
+ATT_MEAN_ABS = 1e-2
+
+
+def f32(x) -> float:
+    """The float32 value of a parameter, as the kernels receive it."""
+    return float(np.float32(x))
+
+
+def layout(seq) -> orc.SeqLayout:
+    return orc.SeqLayout(seq.n_orig, seq.block_start, seq.state, seq.prev_conf, seq.shadow_src)
+
+
+def oracle_attention(wl, layer, seq_index, rows=None, scale=None):
+    """fp64 oracle output [len(rows), hq, d] for one sequence of one layer."""
+    offs = wl.row_offsets()
+    a, b = offs[seq_index], offs[seq_index + 1]
+    lay = layout(wl.seqs[seq_index])
+    mask = orc.attention_mask(lay, rows=rows)
+    q, k, v = wl.q[layer][a:b], wl.k[layer][a:b], wl.v[layer][a:b]
+    return orc.masked_attention(q, k, v, mask, scale=scale, rows=rows)
+
+
+def compare_attention(wl, layer, o_host, sample=None, scale=None, rng=None):
+    """Max/mean abs error over every sequence (all rows, or `sample` rows per sequence
+    including every shadow and block row). Returns (max_abs, mean_abs, rows_checked)."""
+    offs = wl.row_offsets()
+    errs, n = [], 0
+    for si, s in enumerate(wl.seqs):
+        R = s.rows
+        if sample is None or sample >= R:
+            rows = np.arange(R)
+        else:
+            rng = rng or np.random.default_rng(0)
+            must = np.concatenate([np.arange(s.block_start, s.block_start + s.block_len),
+                                   np.arange(s.n_orig, R), [0, R - 1]])
+            extra = rng.choice(R, size=sample, replace=False)
+            rows = np.unique(np.concatenate([must, extra]).astype(np.int64))
+        ref = oracle_attention(wl, layer, si, rows=rows, scale=scale)
+        got = o_host[offs[si] + rows].astype(np.float64)
+        errs.append(np.abs(got - ref).reshape(len(rows), -1))
+        n += len(rows)
+    e = np.concatenate(errs)
+    return float(e.max()), float(e.mean()), n
+
+
+def oracle_scores(wl):
+    """Per-sequence oracle results with the kernels' float32 parameters."""
+    offs = wl.block_offsets()
+    out = []
+    for si, s in enumerate(wl.seqs):
+        a, b = offs[si], offs[si + 1]
+        out.append(orc.score_block(wl.logits_x[a:b], wl.logits_s[a:b], s.state,
+                                   f32(wl.tau_c), f32(wl.tau_u), f32(wl.lam), f32(wl.p0)))
+    return out
+
+
+def compare_scores(wl, conf, token, state_out, w_out=None, counts=None):
+    """Checks the kernel outputs against the oracle. Exact: states and tokens, except rows
+    whose oracle confidence lies within BORDER of a threshold (and, for a C row, the M rows
+    of its block, whose w depends on it) and tokens of rows whose scored logits have a top-2
+    gap under NEAR_TIE. Returns a report dict; raises AssertionError on any mismatch."""
+    offs = wl.block_offsets()
+    taus = (f32(wl.tau_c), f32(wl.tau_u))
+    rep = {"rows": 0, "borderline": 0, "near_tie": 0, "max_conf_err": 0.0, "max_w_ulps": 0.0}
+    for si, (s, res) in enumerate(zip(wl.seqs, oracle_scores(wl))):
+        a, b = offs[si], offs[si + 1]
+        st = np.where(s.state > 2, 0, s.state)
+        border = np.array([min(abs(c - taus[0]), abs(c - taus[1])) < BORDER for c in res.conf])
+        c_border = bool((border & (st == 1)).any())
+        for i in range(b - a):
+            r = a + i
+            rep["rows"] += 1
+            skip_state = border[i] or (st[i] == 0 and c_border)
+            if skip_state:
+                rep["borderline"] += 1
+                continue
+            assert state_out[r] == res.state_out[i], (si, i, state_out[r], res.state_out[i])
+            if st[i] == 0:
+                row = orc.mix_logits(wl.logits_x[r], wl.logits_s[r], res.w[i])
+                if w_out is not None:
+                    ulps = abs(float(w_out[r]) - float(res.w[i])) / float(np.spacing(np.float32(res.w[i])))
+                    rep["max_w_ulps"] = max(rep["max_w_ulps"], ulps)
+                    assert ulps <= 2, (si, i, w_out[r], res.w[i])
+            else:
+                row = wl.logits_s[r]
+                if w_out is not None:
+                    assert np.isnan(w_out[r])
+            tie = res.valid[i] and orc.top2_gap(row) < NEAR_TIE
+            if tie:
+                rep["near_tie"] += 1
+            else:
+                assert token[r] == res.token[i], (si, i, token[r], res.token[i])
+            err = abs(float(conf[r]) - res.conf[i])
+            rep["max_conf_err"] = max(rep["max_conf_err"], err)
+            assert err <= CONF_TOL, (si, i, conf[r], res.conf[i])
+        if counts is not None and not c_border and not border.any():
+            assert list(counts[3 * si:3 * si + 3]) == list(res.counts), (si, counts[3 * si:3 * si + 3], res.counts)
+    return rep

@@ -1,0 +1,121 @@
+"""The C-ABI library builds, loads, exports every symbol of include/dard.h, and rejects bad
+arguments on the host before any launch (no GPU needed: nothing here reaches a kernel)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2608_26574_gb300 import binding as B
+from paper_2608_26574_gb300 import build as BUILD
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    BUILD.build()
+    return B.lib()
+
+
+def _declared_symbols():
+    names = set()
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", f)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(dard_[a-z0-9_]+)\s*\(", text))
+    return names
+
+
+def test_exports_every_declared_symbol(lib):
+    declared = _declared_symbols()
+    assert {"dard_step_attention", "dard_score_and_transition"} <= declared
+    for name in declared:
+        assert hasattr(lib, name), name
+    assert declared <= set(B.EXPORTS)
+
+
+def test_host_only_entry_points(lib):
+    assert lib.dard_version() >= 100
+    assert B.status_string(0) == "DARD_OK"
+    assert B.status_string(7) == "DARD_ERR_WORKSPACE"
+    assert B.status_string(99) == "DARD_ERR_UNKNOWN"
+    assert B.dard_score_workspace_size(32, 126464, 1) > 32 * 64 * 16
+    assert B.dard_score_workspace_size(-1, 10, 1) == 0
+    assert B.dard_score_workspace_size(4, 10, 0) == 0
+
+
+def _attn_args(**kw):
+    n = np.array([64], np.int32)
+    b0 = np.array([32], np.int32)
+    bl = np.array([32], np.int32)
+    sl = np.array([32], np.int32)
+    a = B.AttnArgs()
+    a.q = a.k = a.v = a.o = 0x10000
+    a.dtype, a.hq, a.hkv, a.head_dim, a.num_seqs = B.DARD_BF16, 4, 4, 64, 1
+    keep = {"n": kw.pop("n", n), "b0": kw.pop("b0", b0), "bl": kw.pop("bl", bl), "sl": kw.pop("sl", sl)}
+    a.n_orig = keep["n"].ctypes.data_as(B._I32P)
+    a.block_start = keep["b0"].ctypes.data_as(B._I32P)
+    a.block_len = keep["bl"].ctypes.data_as(B._I32P)
+    a.shadow_len = keep["sl"].ctypes.data_as(B._I32P)
+    a.state = a.prev_conf = a.shadow_src = 0x20000
+    a.scale = 0.0
+    for k, v in kw.items():
+        setattr(a, k, v)
+    return a, keep
+
+
+@pytest.mark.parametrize("change,code", [
+    ({"q": None}, 1), ({"state": None}, 1), ({"shadow_src": None}, 1),
+    ({"dtype": 7}, 3), ({"num_seqs": 0}, 2), ({"num_seqs": 257}, 2),
+    ({"hq": 6, "hkv": 4}, 2), ({"head_dim": 96}, 4), ({"scale": -1.0}, 3),
+    ({"scale": float("inf")}, 3), ({"q": 0x10008}, 6),
+    ({"n": np.array([0], np.int32)}, 2), ({"bl": np.array([129], np.int32)}, 2),
+    ({"b0": np.array([40], np.int32)}, 2), ({"sl": np.array([33], np.int32)}, 2),
+    ({"b0": np.array([-1], np.int32)}, 2),
+])
+def test_attention_validation(lib, change, code):
+    a, keep = _attn_args(**change)
+    assert lib.dard_step_attention(ctypes.byref(a), None) == code
+    assert lib.dard_last_error().decode() != ""
+
+
+def test_attention_null_args(lib):
+    assert lib.dard_step_attention(None, None) == 1
+
+
+def _score_args(**kw):
+    bl = kw.pop("bl", np.array([32], np.int32))
+    a = B.ScoreArgs()
+    a.logits_x = a.logits_s = 0x10000
+    a.dtype, a.vocab, a.row_stride, a.num_seqs = B.DARD_BF16, 1024, 1024, 1
+    a.block_len = bl.ctypes.data_as(B._I32P)
+    a.state_in = 0x20000
+    a.tau_c, a.tau_u, a.lambda_, a.p0 = 0.5, 0.8, 0.917, 0.1
+    a.conf = a.token = a.state_out = 0x30000
+    a.workspace = 0x40000
+    a.workspace_bytes = 1 << 20
+    for k, v in kw.items():
+        setattr(a, k, v)
+    return a, bl
+
+
+@pytest.mark.parametrize("change,code", [
+    ({"logits_s": None}, 1), ({"conf": None}, 1), ({"state_in": None}, 1),
+    ({"dtype": 3}, 3), ({"vocab": 0}, 2), ({"row_stride": 100}, 2),
+    ({"tau_c": 0.9, "tau_u": 0.8}, 3), ({"tau_u": 1.5}, 3), ({"lambda_": 1.0}, 3),
+    ({"lambda_": 0.0}, 3), ({"p0": 0.0}, 3), ({"num_seqs": 0}, 2),
+    ({"bl": np.array([200], np.int32)}, 2), ({"workspace": None}, 7),
+    ({"workspace_bytes": 16}, 7), ({"logits_x": 0x10002}, 6), ({"row_stride": 1025}, 6),
+])
+def test_score_validation(lib, change, code):
+    a, keep = _score_args(**change)
+    assert lib.dard_score_and_transition(ctypes.byref(a), None) == code
+
+
+def test_binding_raises_without_library(tmp_path, monkeypatch):
+    monkeypatch.setattr(B, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        B.lib(str(tmp_path / "libdard.so"))

@@ -1,0 +1,129 @@
+"""GPU parity of dard_step_attention against the CPU oracle (Eq. 2-3, Sec. 3.2 blocks 1-6)."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_26574_gb300 import workloads as W
+from paper_2608_26574_gb300.device import DeviceStep
+
+from . import parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+def _attend(wl, layer=0, scale=0.0):
+    ds = DeviceStep(wl, layers=[layer], scoring=False)
+    o = ds.attention(0, scale=scale)
+    torch.cuda.synchronize()
+    return ds, o.float().cpu().numpy()
+
+
+@pytest.mark.parametrize("name,layout,sample", [
+    ("tiny", "paper", None), ("tiny", "candidates", None),
+    ("8b", "paper", None), ("8b", "candidates", None),
+    ("gqa", "paper", 192), ("gqa", "candidates", 192),
+    ("ragged", "paper", 48), ("mm", "paper", 64),
+])
+def test_attention_configs(name, layout, sample):
+    wl = W.make(name, layout=layout, scoring=False, layers=2 if name == "mm" else None)
+    layers = [0, 1] if name == "mm" else [0]
+    for li in layers:
+        ds, o = _attend(wl, li)
+        mx, mean, n = P.compare_attention(wl, li, o, sample=sample)
+        print(name, layout, li, "max", mx, "mean", mean, "rows", n)
+        assert mx <= P.ATT_MAX_ABS and mean <= P.ATT_MEAN_ABS
+        assert int(ds.status.item()) == 0
+
+
+def _probe_tol(wl):
+    # Q = 0: every attended key has weight 1/N, so a single wrong key moves the output by
+    # |v_a - v_b| / N >> this tolerance (bf16 output rounding and fp32 sums stay far below)
+    n_min = min(s.n_orig for s in wl.seqs)
+    return 0.25 / n_min
+
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("layout", ["paper", "candidates"])
+def test_mask_probe_every_key(d, layout):
+    """Uniform attention (Q = 0) exposes every key selection of the in-kernel mask."""
+    specs = [dict(n_orig=200, block_start=100, block_len=64, fractions=(0.3, 0.4, 0.3),
+                  shadow=layout),
+             dict(n_orig=131, block_start=0, block_len=37, fractions=(0.2, 0.5, 0.3), shadow=layout),
+             dict(n_orig=97, block_start=60, block_len=37, fractions=(0.5, 0.3, 0.2), shadow=layout),
+             dict(n_orig=300, block_start=172, block_len=128, fractions=(0.3, 0.4, 0.3),
+                  shadow=layout)]
+    wl = W.custom(specs, 4, 2, d, probe=True, seed=21 + d)
+    ds, o = _attend(wl)
+    mx, mean, n = P.compare_attention(wl, 0, o)
+    print("probe", d, layout, mx, mean, n)
+    assert mx <= _probe_tol(wl)
+
+
+def test_mask_probe_confidence_ties():
+    """Equal c_{t-1} among C tokens attend each other both ways (Eq. 3 uses <=)."""
+    B = 48
+    st = np.array([1] * 24 + [0] * 12 + [2] * 12, dtype=np.uint8)
+    np.random.default_rng(0).shuffle(st)
+    cf = np.where(st == 1, np.float32(0.65), np.float32(0.2)).astype(np.float32)
+    cf[st == 2] = 0.95
+    cf[np.flatnonzero(st == 1)[:8]] = 0.7
+    specs = [dict(n_orig=160, block_start=70, state=st, prev_conf=cf)]
+    wl = W.custom(specs, 2, 2, 128, probe=True, seed=5)
+    _, o = _attend(wl)
+    mx, _, _ = P.compare_attention(wl, 0, o)
+    assert mx <= _probe_tol(wl)
+
+
+@pytest.mark.parametrize("states", ["M", "C", "U"])
+def test_mask_probe_uniform_states(states):
+    code = {"M": 0, "C": 1, "U": 2}[states]
+    specs = [dict(n_orig=256, block_start=128, state=np.full(64, code, np.uint8))]
+    wl = W.custom(specs, 2, 1, 128, probe=True, seed=code)
+    _, o = _attend(wl)
+    mx, _, _ = P.compare_attention(wl, 0, o)
+    assert mx <= _probe_tol(wl)
+
+
+@pytest.mark.parametrize("case", range(12))
+def test_attention_random_shapes(case):
+    """Seeded random ragged batches: odd lengths, blocks at the start / end, S = 0,
+    B = 1..128, grouped heads, larger scores (scale up to 1) to exercise the O rescale."""
+    rng = np.random.default_rng(100 + case)
+    specs = []
+    for _ in range(int(rng.integers(1, 5))):
+        n = int(rng.integers(1, 700))
+        B = int(rng.integers(0, min(n, 128) + 1))
+        b0 = int(rng.integers(0, n - B + 1))
+        shadow = ["paper", "candidates", "none"][int(rng.integers(0, 3))]
+        sp = dict(n_orig=n, block_start=b0, block_len=B,
+                  fractions=tuple(rng.dirichlet([1, 1, 1])))
+        sp["shadow"] = np.zeros(0, np.int32) if shadow == "none" else shadow
+        specs.append(sp)
+    hkv = int(rng.choice([1, 2, 4]))
+    hq = hkv * int(rng.choice([1, 2, 3]))
+    d = int(rng.choice([64, 128]))
+    std = float(rng.choice([1.0 / np.sqrt(d), 0.5, 1.0]))
+    wl = W.custom(specs, hq, hkv, d, seed=200 + case, qkv_std=std)
+    scale = float(rng.choice([0.0, 0.3, 1.0]))
+    ds, o = _attend(wl, scale=scale)
+    mx, mean, n = P.compare_attention(wl, 0, o, scale=scale or None)
+    print(case, [(s.n_orig, s.block_start, s.block_len, s.n_shadow) for s in wl.seqs],
+          hq, hkv, d, std, scale, mx, mean)
+    assert mx <= P.ATT_MAX_ABS and mean <= P.ATT_MEAN_ABS
+
+
+def test_attention_bad_shadow_rows_flagged():
+    """shadow_src outside the block or repeated: status bit, other rows still correct."""
+    specs = [dict(n_orig=128, block_start=32, block_len=16, fractions=(0.4, 0.3, 0.3),
+                  shadow=np.array([32, 33, 34, 34, 90, 35], np.int32))]
+    wl = W.custom(specs, 2, 2, 128, seed=3)
+    ds, o = _attend(wl)
+    assert int(ds.status.item()) & 0x2
+    # rows 0..127 of x: the oracle with the two bad shadow rows removed
+    good = W.custom([dict(n_orig=128, block_start=32, state=wl.seqs[0].state,
+                          prev_conf=wl.seqs[0].prev_conf, shadow=np.array([32, 33, 34, 35], np.int32))],
+                    2, 2, 128, seed=3)
+    keep = np.r_[0:128, 128, 129, 130, 133]
+    good.q[0], good.k[0], good.v[0] = wl.q[0][keep], wl.k[0][keep], wl.v[0][keep]
+    ref = P.oracle_attention(good, 0, 0)
+    np.testing.assert_allclose(o[keep], ref, atol=P.ATT_MAX_ABS)

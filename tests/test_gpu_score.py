@@ -1,0 +1,105 @@
+"""GPU parity of dard_score_and_transition against the CPU oracle (Eq. 1, 5-8, Algorithm 1)."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_26574_gb300 import workloads as W
+from paper_2608_26574_gb300.device import DeviceStep
+
+from . import parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(wl, state_in=None, reps=1):
+    ds = DeviceStep(wl, attention=False)
+    for _ in range(reps):
+        ds.score(state_in=state_in)
+    torch.cuda.synchronize()
+    return ds, (ds.conf.cpu().numpy(), ds.token.cpu().numpy(), ds.state_out.cpu().numpy(),
+                ds.w_out.cpu().numpy(), ds.counts.cpu().numpy())
+
+
+def _check(wl, outs):
+    conf, token, st, w, counts = outs
+    rep = P.compare_scores(wl, conf, token, st, w_out=w, counts=counts)
+    offs = wl.block_offsets()
+    for si in range(len(wl.seqs)):
+        want = np.bincount(st[offs[si]:offs[si + 1]], minlength=3)
+        assert list(counts[3 * si:3 * si + 3]) == list(want)
+    return rep
+
+
+@pytest.mark.parametrize("name", ["tiny", "8b", "gqa", "ragged", "mm"])
+@pytest.mark.parametrize("mode", ["literal", "spanning"])
+def test_score_configs(name, mode):
+    wl = W.make(name, logits=mode, attention=False)
+    ds, outs = _run(wl)
+    rep = _check(wl, outs)
+    assert int(ds.status.item()) == 0
+    print(name, mode, rep)
+
+
+def test_score_twice_in_a_row_same_result():
+    """The workspace counters return to zero: a second call gives identical outputs."""
+    wl = W.make("8b", logits="spanning", attention=False)
+    ds = DeviceStep(wl, attention=False)
+    ds.score()
+    first = [t.clone() for t in (ds.conf, ds.token, ds.state_out, ds.w_out, ds.counts)]
+    ds.score()
+    torch.cuda.synchronize()
+    for a, b in zip(first, (ds.conf, ds.token, ds.state_out, ds.w_out, ds.counts)):
+        assert torch.equal(a, b) or bool(((a == b) | (torch.isnan(a) & torch.isnan(b))).all())
+
+
+@pytest.mark.parametrize("vocab", [1, 7, 8, 9, 1000, 2049, 8191, 65537])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_score_ragged_vocab_tails(vocab, dtype):
+    specs = [dict(n_orig=40, block_start=8, block_len=24, fractions=(0.4, 0.3, 0.3))]
+    wl = W.custom(specs, 1, 1, 64, dtype=dtype, vocab=vocab, seed=vocab, logit_std=2.0)
+    _check(wl, _run(wl)[1])
+
+
+def test_score_many_sequences_and_degenerate_blocks():
+    specs = [dict(n_orig=300, block_start=100, block_len=B, fractions=f)
+             for B, f in ((1, (0, 1, 0)), (7, (1, 0, 0)), (32, (0, 0, 1)), (64, (0, 1, 0)),
+                          (128, (0.2, 0.5, 0.3)), (0, (1, 0, 0)), (5, (0.2, 0.4, 0.4)))]
+    wl = W.custom(specs, 1, 1, 64, vocab=5000, seed=3)
+    _check(wl, _run(wl)[1])
+
+
+def test_score_exact_ties_lowest_index():
+    specs = [dict(n_orig=64, block_start=0, block_len=16, fractions=(0.5, 0.25, 0.25))]
+    wl = W.custom(specs, 1, 1, 64, vocab=4096, seed=5, logits="plain")
+    # plant the same maximum at several columns of every row (bf16-exact values)
+    for arr in (wl.logits_x, wl.logits_s):
+        for r in range(arr.shape[0]):
+            cols = np.sort(np.random.default_rng(r).choice(4096, size=4, replace=False))
+            arr[r, cols] = 16.0
+    conf, token, st, w, counts = _run(wl)[1]
+    _check(wl, (conf, token, st, w, counts))
+
+
+def test_score_nonfinite_rows_and_bad_states():
+    specs = [dict(n_orig=64, block_start=16, state=[0, 1, 2, 0, 1, 2, 7, 1, 0, 2])]
+    wl = W.custom(specs, 1, 1, 64, vocab=3000, seed=9)
+    wl.logits_s[1, 17] = np.nan          # C row with a NaN -> invalid
+    wl.logits_s[2, 5] = np.inf           # U row with +inf -> invalid
+    wl.logits_s[4, :] = -np.inf          # C row all -inf -> invalid
+    wl.logits_x[3, 100] = np.nan         # M row: NaN in the original logits
+    wl.logits_s[5, :10] = -np.inf        # some -inf values are fine
+    ds, outs = _run(wl)
+    conf, token, st, w, counts = outs
+    _check(wl, outs)
+    for r in (1, 2, 3, 4):
+        assert conf[r] == 0 and token[r] == -1 and st[r] == 0
+    s = int(ds.status.item())
+    assert s & 0x4 and s & 0x1   # invalid rows and the state byte 7
+
+
+def test_score_threshold_edges():
+    """tau_c == tau_u (two states only) and the extreme thresholds 0 and 1."""
+    specs = [dict(n_orig=80, block_start=40, block_len=32, fractions=(0.4, 0.3, 0.3))]
+    for tau in ((0.6, 0.6), (0.0, 1.0), (0.0, 0.0), (1.0, 1.0)):
+        wl = W.custom(specs, 1, 1, 64, vocab=2000, seed=11, tau=tau, logit_std=1.0)
+        _check(wl, _run(wl)[1])

@@ -271,7 +271,9 @@ def test_masked_attention_matches_library_sdpa_with_dense_mask():
         want = _sdpa_torch(q, k, v, mask=mask, scale=scale)
         np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
     rows = np.array([0, 3, R - 1])
-    np.testing.assert_allclose(orc.masked_attention(q, k, v, mask, rows=rows),
+    sub = orc.attention_mask(lay, rows=rows)
+    assert (sub == mask[rows]).all()
+    np.testing.assert_allclose(orc.masked_attention(q, k, v, sub, rows=rows),
                                orc.masked_attention(q, k, v, mask)[rows], atol=0)
 
 
