@@ -100,6 +100,15 @@ def _ptr(t) -> int | None:
     return t.data_ptr()
 
 
+def _rows_ptr(t) -> int:
+    """Device pointer of a 2-D tensor whose rows are contiguous (any row pitch)."""
+    if not t.is_cuda:
+        raise ValueError("device tensor expected")
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("2-D tensor with contiguous rows expected")
+    return t.data_ptr()
+
+
 def _host_i32(a) -> np.ndarray:
     return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
 
@@ -146,10 +155,13 @@ def dard_score_workspace_size(rows: int, vocab: int, num_seqs: int) -> int:
 def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, tau_u, lam, p0,
                               conf, token, state_out, workspace, w_out=None, counts=None,
                               status=None, stream=None):
-    """Scoring and transition of every block row; logits [rows, V] (row stride V)."""
+    """Scoring and transition of every block row; logits [rows, V] with contiguous rows and
+    the same row pitch (``stride(0)``, at least V) in both tensors."""
     block_len = _host_i32(block_len)
+    if logits_x.stride(0) != logits_s.stride(0) or logits_x.shape != logits_s.shape:
+        raise ValueError("logits_x and logits_s need the same shape and row pitch")
     a = ScoreArgs()
-    a.logits_x, a.logits_s = _ptr(logits_x), _ptr(logits_s)
+    a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
     a.dtype = _dtype_code(logits_s)
     a.vocab = logits_s.shape[1]
     a.row_stride = logits_s.stride(0)

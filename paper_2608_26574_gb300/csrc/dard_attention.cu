@@ -36,9 +36,8 @@ namespace dard {
 namespace {
 
 constexpr int kBM = 128;  // query rows per CTA
-constexpr int kBN = 128;  // keys per tile
 constexpr int kTcThreads = 192;
-constexpr uint32_t kTmemCols = 256;  // S/P: columns [0,128), O: [128, 128 + D)
+constexpr uint32_t kTmemCols = 256;  // S/P buffers: columns [0,64), [64,128); O: [128, 128 + D)
 constexpr float kRescaleLog2 = 8.0f;
 
 // Per-CTA copy of the current block: states, confidences and the shadow maps.
@@ -156,9 +155,71 @@ __device__ __forceinline__ bool key_visible(const RowInfo& q, const BlockInfo& b
   return true;
 }
 
+// ---------------------------------------------------------------- tensor-core path
+// Row masks over block positions (bit j = block position j), or over shadow rows.
+struct Bits128 {
+  uint64_t lo, hi;
+};
+
+__device__ __forceinline__ void set_bit(Bits128& b, int j) {
+  if (j < 64) b.lo |= 1ull << j; else b.hi |= 1ull << (j - 64);
+}
+__device__ __forceinline__ bool get_bit(const Bits128& b, int j) {
+  return ((j < 64 ? b.lo >> j : b.hi >> (j - 64)) & 1ull) != 0;
+}
+// 64 bits of b starting at bit `start` (0 <= start); bits past 127 read as 0.
+__device__ __forceinline__ uint64_t bits_window(const Bits128& b, int start) {
+  if (start >= 128) return 0;
+  if (start >= 64) return b.hi >> (start - 64);
+  if (start == 0) return b.lo;
+  return (b.lo >> start) | (b.hi << (64 - start));
+}
+
+// Per query row, the two masks the tiles need: block positions whose x copy the row does
+// not see (it takes the shadow copy and the position has one), and shadow rows it sees.
+struct RowMasks {
+  Bits128 hide_x;
+  Bits128 see_s;
+};
+
+__device__ RowMasks row_masks(const RowInfo& q, const BlockInfo& bi, const SeqDesc& sd) {
+  Bits128 ts{0, 0};  // takes_shadow for every block position
+  for (int j = 0; j < sd.blen; ++j)
+    if (takes_shadow(q, bi.st[j], bi.cf[j], j)) set_bit(ts, j);
+  RowMasks m{{0, 0}, {0, 0}};
+  for (int j = 0; j < sd.blen; ++j)
+    if (bi.shrow[j] >= 0 && get_bit(ts, j)) set_bit(m.hide_x, j);
+  for (int k = 0; k < sd.slen; ++k) {
+    const int j = bi.shpos[k];
+    if (j >= 0 && get_bit(ts, j)) set_bit(m.see_s, k);
+  }
+  return m;
+}
+
+constexpr int kTN = 64;  // keys per tile of the tensor-core path
+
 __device__ __forceinline__ bool tile_needs_mask(const SeqDesc& sd, int kt0) {
-  return (kt0 + kBN > sd.n_orig) ||
-         (sd.blen > 0 && kt0 < sd.b0 + sd.blen && kt0 + kBN > sd.b0);
+  return (kt0 + kTN > sd.n_orig) ||
+         (sd.blen > 0 && kt0 < sd.b0 + sd.blen && kt0 + kTN > sd.b0);
+}
+
+// Visibility of keys [kt0, kt0 + 64) for one row (bit t = key kt0 + t).
+__device__ __forceinline__ uint64_t tile_visibility(const SeqDesc& sd, int kt0, const RowMasks& m) {
+  uint64_t vis = ~0ull;
+  const int lo = max(kt0, sd.b0), hi = min(kt0 + kTN, sd.b0 + sd.blen);
+  if (lo < hi) {
+    const int len = hi - lo;
+    uint64_t h = bits_window(m.hide_x, lo - sd.b0);
+    if (len < 64) h &= (1ull << len) - 1;
+    vis &= ~(h << (lo - kt0));
+  }
+  if (kt0 + kTN > sd.n_orig) {
+    const int s_lo = max(kt0, sd.n_orig);
+    const int off = s_lo - kt0;  // 0..63
+    const uint64_t keep = off == 0 ? 0ull : ((1ull << off) - 1);
+    vis = (vis & keep) | (bits_window(m.see_s, s_lo - sd.n_orig) << off);
+  }
+  return vis;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -167,8 +228,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+// Every barrier below completes one phase per use; a waiter is never more than one phase
+// behind the phase it waits for (the parity would alias otherwise). PV completion is
+// therefore tracked per S/P buffer (pv_done[b]: tiles b, b+2, ...), and the end of the
+// last PV by its own single-phase barrier o_full.
 struct __align__(8) TcCtl {
-  uint64_t q_full, k_full, k_empty, v_full, v_empty, s_full, p_full, pv_done;
+  uint64_t q_full, o_full;
+  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], p_full[2], pv_done[2];
   uint32_t tmem_base;
   int32_t abort;
   BlockInfo bi;
@@ -176,7 +242,9 @@ struct __align__(8) TcCtl {
 
 template <int D>
 constexpr size_t tc_smem_bytes() {
-  return 1024 /*alignment slack*/ + 3 * static_cast<size_t>(kBM) * D * 2 + sizeof(TcCtl);
+  // alignment slack + Q (128 rows) + two stages each of K and V (64 rows) + control
+  return 1024 + static_cast<size_t>(kBM) * D * 2 + 4 * static_cast<size_t>(kTN) * D * 2 +
+         sizeof(TcCtl);
 }
 
 __device__ __forceinline__ void flag_timeout(const AttnParams& p, TcCtl& ctl) {
@@ -188,35 +256,40 @@ template <int D>
 __global__ void __launch_bounds__(kTcThreads, 2)
     attn_tc(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmq,
             const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv) {
-  constexpr int kSub = D / 64;                    // 128-byte (64 x bf16) column blocks
-  constexpr uint32_t kSubBytes = kBM * 128;       // one 128-row x 128-byte swizzled block
-  constexpr uint32_t kTileBytes = kSub * kSubBytes;
+  constexpr int kSub = D / 64;                 // 128-byte (64 x bf16) column blocks
+  constexpr uint32_t kQSub = kBM * 128;        // one 128-row x 128-byte swizzled block
+  constexpr uint32_t kKSub = kTN * 128;        // one 64-row x 128-byte swizzled block
+  constexpr uint32_t kQBytes = kSub * kQSub;
+  constexpr uint32_t kKVBytes = kSub * kKSub;  // one K (or V) tile of 64 keys
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sQ = base;
-  uint8_t* sK = sQ + kTileBytes;
-  uint8_t* sV = sK + kTileBytes;
-  TcCtl& ctl = *reinterpret_cast<TcCtl*>(sV + kTileBytes);
+  uint8_t* sK = sQ + kQBytes;        // stages at sK, sK + kKVBytes
+  uint8_t* sV = sK + 2 * kKVBytes;   // stages at sV, sV + kKVBytes
+  TcCtl& ctl = *reinterpret_cast<TcCtl*>(sV + 2 * kKVBytes);
 
   int seq, qt, h;
   decode_work(p, blockIdx.x, seq, qt, h);
   const SeqDesc sd = p.seq[seq];
   const int rows_seq = sd.n_orig + sd.slen;
-  const int n_kt = (rows_seq + kBN - 1) / kBN;
+  const int n_kt = (rows_seq + kTN - 1) / kTN;
   const int q0 = qt * kBM;
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(&ctl.q_full, 1);
-    mbar_init(&ctl.k_full, 1);
-    mbar_init(&ctl.k_empty, 1);
-    mbar_init(&ctl.v_full, 1);
-    mbar_init(&ctl.v_empty, 1);
-    mbar_init(&ctl.s_full, 1);
-    mbar_init(&ctl.p_full, 4);
-    mbar_init(&ctl.pv_done, 1);
+    mbar_init(&ctl.o_full, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&ctl.pv_done[b], 1);
+      mbar_init(&ctl.k_full[b], 1);
+      mbar_init(&ctl.k_empty[b], 1);
+      mbar_init(&ctl.v_full[b], 1);
+      mbar_init(&ctl.v_empty[b], 1);
+      mbar_init(&ctl.s_full[b], 1);
+      mbar_init(&ctl.p_full[b], 4);
+    }
     ctl.abort = 0;
     fence_barrier_init();
   }
@@ -228,7 +301,6 @@ __global__ void __launch_bounds__(kTcThreads, 2)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tS = ctl.tmem_base;
   const uint32_t tO = ctl.tmem_base + 128;
   volatile int32_t* abort_flag = &ctl.abort;
 
@@ -239,61 +311,76 @@ __global__ void __launch_bounds__(kTcThreads, 2)
       tma_prefetch_desc(&tmk);
       tma_prefetch_desc(&tmv);
       const int row0 = sd.row_base;
-      mbar_arrive_expect_tx(&ctl.q_full, kTileBytes);
+      mbar_arrive_expect_tx(&ctl.q_full, kQBytes);
 #pragma unroll
       for (int s = 0; s < kSub; ++s)
-        tma_load_2d(sQ + s * kSubBytes, &tmq, &ctl.q_full, h * D + s * 64, row0 + q0);
-      int issued = 0;
+        tma_load_2d(sQ + s * kQSub, &tmq, &ctl.q_full, h * D + s * 64, row0 + q0);
+      int last_k = -1, last_v = -1;
       for (int j = 0; j < n_kt && !*abort_flag; ++j) {
-        if (j > 0 && !mbar_wait(&ctl.k_empty, (j - 1) & 1)) { flag_timeout(p, ctl); break; }
-        mbar_arrive_expect_tx(&ctl.k_full, kTileBytes);
+        const int b = j & 1;
+        if (j >= 2 && !mbar_wait(&ctl.k_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
+        mbar_arrive_expect_tx(&ctl.k_full[b], kKVBytes);
 #pragma unroll
         for (int s = 0; s < kSub; ++s)
-          tma_load_2d(sK + s * kSubBytes, &tmk, &ctl.k_full, g * D + s * 64, row0 + j * kBN);
-        if (j > 0 && !mbar_wait(&ctl.v_empty, (j - 1) & 1)) { flag_timeout(p, ctl); issued = 2 * j + 1; break; }
-        mbar_arrive_expect_tx(&ctl.v_full, kTileBytes);
+          tma_load_2d(sK + b * kKVBytes + s * kKSub, &tmk, &ctl.k_full[b], g * D + s * 64,
+                      row0 + j * kTN);
+        last_k = j;
+        if (j >= 2 && !mbar_wait(&ctl.v_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
+        mbar_arrive_expect_tx(&ctl.v_full[b], kKVBytes);
 #pragma unroll
         for (int s = 0; s < kSub; ++s)
-          tma_load_2d(sV + s * kSubBytes, &tmv, &ctl.v_full, g * D + s * 64, row0 + j * kBN);
-        issued = 2 * j + 2;
+          tma_load_2d(sV + b * kKVBytes + s * kKSub, &tmv, &ctl.v_full[b], g * D + s * 64,
+                      row0 + j * kTN);
+        last_v = j;
       }
-      if (*abort_flag && issued > 0) {
-        // let the copies already in flight land before the CTA's shared memory is released
-        const int jk = (issued - 1) / 2;
-        mbar_wait(&ctl.k_full, jk & 1);
-        if ((issued & 1) == 0) mbar_wait(&ctl.v_full, jk & 1);
+      if (*abort_flag) {
+        // let the copies already in flight land before shared memory is released
+        if (last_k >= 0) mbar_wait(&ctl.k_full[last_k & 1], (last_k >> 1) & 1);
+        if (last_v >= 0) mbar_wait(&ctl.v_full[last_v & 1], (last_v >> 1) & 1);
       }
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kBN, 0, 0);
+      constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
       const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK), av = smem_u32(sV);
-      bool ok = mbar_wait(&ctl.q_full, 0);
-      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
-        ok = mbar_wait(&ctl.k_full, j & 1);
-        if (ok && j > 0) ok = mbar_wait(&ctl.pv_done, (j - 1) & 1);
-        if (!ok) break;
+      auto issue_s = [&](int t) -> bool {  // S_t = Q K_t^T into S buffer t & 1
+        const int b = t & 1;
+        if (!mbar_wait(&ctl.k_full[b], (t >> 1) & 1)) return false;
         tc_fence_after();
+        const uint32_t kb = ak + b * kKVBytes;
 #pragma unroll
         for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t off = (ks >> 2) * kSubBytes + (ks & 3) * 32;
-          mma_ss(tS, smem_desc_sw128(aq + off, 16, 1024), smem_desc_sw128(ak + off, 16, 1024),
-                 kIdS, ks > 0);
+          const uint32_t qo = (ks >> 2) * kQSub + (ks & 3) * 32;
+          const uint32_t ko = (ks >> 2) * kKSub + (ks & 3) * 32;
+          mma_ss(ctl.tmem_base + b * kTN, smem_desc_sw128(aq + qo, 16, 1024),
+                 smem_desc_sw128(kb + ko, 16, 1024), kIdS, ks > 0);
         }
-        mma_commit(&ctl.s_full);
-        mma_commit(&ctl.k_empty);
-        ok = mbar_wait(&ctl.p_full, j & 1);
-        if (ok) ok = mbar_wait(&ctl.v_full, j & 1);
+        mma_commit(&ctl.s_full[b]);
+        mma_commit(&ctl.k_empty[b]);
+        return true;
+      };
+      bool ok = mbar_wait(&ctl.q_full, 0);
+      if (ok) ok = issue_s(0);
+      if (ok && n_kt > 1) ok = issue_s(1);
+      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
+        const int b = j & 1;
+        ok = mbar_wait(&ctl.p_full[b], (j >> 1) & 1) && mbar_wait(&ctl.v_full[b], (j >> 1) & 1);
         if (!ok) break;
         tc_fence_after();
+        const uint32_t vb = av + b * kKVBytes;
 #pragma unroll
-        for (int ks = 0; ks < kBN / 16; ++ks)
-          mma_ts(tO, tS + ks * 8, smem_desc_sw128(av + ks * 2048, kSubBytes, 1024), kIdO,
-                 (j > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&ctl.pv_done);
-        mma_commit(&ctl.v_empty);
+        for (int ks = 0; ks < kTN / 16; ++ks)
+          mma_ts(tO, ctl.tmem_base + b * kTN + ks * 8,
+                 smem_desc_sw128(vb + ks * 2048, kKSub, 1024), kIdO, (j > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&ctl.pv_done[b]);
+        mma_commit(&ctl.v_empty[b]);
+        if (j == n_kt - 1) mma_commit(&ctl.o_full);
+        if (j + 2 < n_kt) {
+          // S buffer b is free once PV_j has read P_j out of it
+          ok = mbar_wait(&ctl.pv_done[b], (j >> 1) & 1) && issue_s(j + 2);
+        }
       }
       if (!ok) flag_timeout(p, ctl);
     }
@@ -301,49 +388,52 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     // ------------------------------------------------------------ softmax + epilogue
     const int t = threadIdx.x;
     const RowInfo q = row_info(sd, ctl.bi, q0 + t);
+    const RowMasks rm = row_masks(q, ctl.bi, sd);
     const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
     const float sl = p.scale_log2;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < n_kt; ++j) {
-      const int kt0 = j * kBN;
-      uint32_t vis[4] = {~0u, ~0u, ~0u, ~0u};
+      const int b = j & 1;
+      const int kt0 = j * kTN;
       const bool masked = tile_needs_mask(sd, kt0);
-      if (masked) {
-        for (int k = 0; k < kBN; ++k)
-          if (!key_visible(q, ctl.bi, sd, kt0 + k)) vis[k >> 5] &= ~(1u << (k & 31));
-      }
-      ok = !*abort_flag && mbar_wait(&ctl.s_full, j & 1);
+      const uint64_t vis = masked ? tile_visibility(sd, kt0, rm) : ~0ull;
+      ok = !*abort_flag && mbar_wait(&ctl.s_full[b], (j >> 1) & 1);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
-      float s[kBN];
+      uint32_t r0[32], r1[32];
+      tmem_ld32(ctl.tmem_base + b * kTN + lane_off, r0);
+      tmem_ld32(ctl.tmem_base + b * kTN + 32 + lane_off, r1);
+      tmem_wait_ld();
+      float s[kTN];
 #pragma unroll
-      for (int c = 0; c < kBN / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tS + lane_off + c * 32, r);
-        tmem_wait_ld();
-#pragma unroll
-        for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(r[e]);
+      for (int e = 0; e < 32; ++e) {
+        s[e] = __uint_as_float(r0[e]);
+        s[32 + e] = __uint_as_float(r1[e]);
       }
       float mt = -INFINITY;
       if (masked) {
 #pragma unroll
-        for (int k = 0; k < kBN; ++k) {
-          s[k] = ((vis[k >> 5] >> (k & 31)) & 1u) ? s[k] : -INFINITY;
+        for (int k = 0; k < kTN; ++k) {
+          s[k] = ((vis >> k) & 1ull) ? s[k] : -INFINITY;
           mt = fmaxf(mt, s[k]);
         }
       } else {
 #pragma unroll
-        for (int k = 0; k < kBN; ++k) mt = fmaxf(mt, s[k]);
+        for (int k = 0; k < kTN; ++k) mt = fmaxf(mt, s[k]);
       }
       // Raise the reference maximum on the first finite value, or when the tile maximum
-      // exceeds it by more than 2^kRescaleLog2 in probability; O is rescaled only then.
+      // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
       float m_new = m_run;
       if (m_run == -INFINITY) m_new = mt;
       else if ((mt - m_run) * sl > kRescaleLog2) m_new = mt;
       const bool rescale = (m_new != m_run) && (m_run != -INFINITY);
       const float alpha = rescale ? ex2_approx((m_run - m_new) * sl) : 1.f;
       if (__any_sync(0xffffffffu, rescale)) {
+        // PV_{j-1} may still be accumulating into O: wait for it first
+        ok = mbar_wait(&ctl.pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        tc_fence_after();
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           uint32_t r[32];
@@ -357,24 +447,21 @@ __global__ void __launch_bounds__(kTcThreads, 2)
       l_run *= alpha;
       m_run = m_new;
       const float mL = (m_run == -INFINITY) ? 0.f : m_run * sl;
+      uint32_t pk[32];
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        uint32_t pk[32];
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const float a = ex2_approx(fmaf(s[half * 64 + 2 * e], sl, -mL));
-          const float b = ex2_approx(fmaf(s[half * 64 + 2 * e + 1], sl, -mL));
-          l_run += a + b;
-          pk[e] = pack_bf16x2(a, b);
-        }
-        tmem_st32(tS + lane_off + half * 32, pk);
+      for (int e = 0; e < 32; ++e) {
+        const float a = ex2_approx(fmaf(s[2 * e], sl, -mL));
+        const float c = ex2_approx(fmaf(s[2 * e + 1], sl, -mL));
+        l_run += a + c;
+        pk[e] = pack_bf16x2(a, c);
       }
+      tmem_st32(ctl.tmem_base + b * kTN + lane_off, pk);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.p_full);
+      if (lane == 0) mbar_arrive(&ctl.p_full[b]);
     }
-    if (ok) ok = mbar_wait(&ctl.pv_done, (n_kt - 1) & 1);
+    if (ok) ok = mbar_wait(&ctl.o_full, 0);
     if (!__all_sync(0xffffffffu, ok)) {
       if (lane == 0) flag_timeout(p, ctl);
     } else {
@@ -390,15 +477,15 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         tmem_ld32(tO + lane_off + c * 32, rr);
         tmem_wait_ld();
         if (store) {
-          uint32_t pk[16];
+          uint32_t o2[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e)
-            pk[e] = pack_bf16x2(__uint_as_float(rr[2 * e]) * inv_l,
+            o2[e] = pack_bf16x2(__uint_as_float(rr[2 * e]) * inv_l,
                                 __uint_as_float(rr[2 * e + 1]) * inv_l);
           uint4* dst = reinterpret_cast<uint4*>(out + c * 32);
 #pragma unroll
           for (int v = 0; v < 4; ++v)
-            dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+            dst[v] = make_uint4(o2[4 * v], o2[4 * v + 1], o2[4 * v + 2], o2[4 * v + 3]);
         }
       }
     }
@@ -479,12 +566,12 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-bool make_map(CUtensorMap* m, const void* ptr, int heads, int d, int rows) {
+bool make_map(CUtensorMap* m, const void* ptr, int heads, int d, int rows, int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(heads) * d, static_cast<cuuint64_t>(rows)};
   const cuuint64_t strides[1] = {static_cast<cuuint64_t>(heads) * d * 2};
-  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kBM)};
+  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
   const cuuint32_t estr[2] = {1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -511,8 +598,9 @@ template <int D>
 cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
   static std::atomic<uint64_t> attr_done{0};
   CUtensorMap mq, mk, mv;
-  if (!make_map(&mq, p.q, p.hq, D, p.total_rows) || !make_map(&mk, p.k, p.hkv, D, p.total_rows) ||
-      !make_map(&mv, p.v, p.hkv, D, p.total_rows))
+  if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM) ||
+      !make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
+      !make_map(&mv, p.v, p.hkv, D, p.total_rows, kTN))
     return cudaErrorInvalidValue;
   const size_t smem = tc_smem_bytes<D>();
   cudaError_t e = ensure_smem_attr(attn_tc<D>, smem, attr_done);

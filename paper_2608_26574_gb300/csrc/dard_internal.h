@@ -66,6 +66,7 @@ struct ScoreParams {
   int64_t row_stride;
   int32_t vocab, rows, num_seqs, nsplit, chunk;
   float tau_c, tau_u, lambda, p0;
+  double lam_pow[DARD_MAX_BLOCK];  // lambda^k, k = 0 .. DARD_MAX_BLOCK - 1 (Eq. 5 kernel)
   int32_t blk_off[DARD_MAX_SEQS + 1];
 };
 

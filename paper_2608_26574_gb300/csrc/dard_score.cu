@@ -16,6 +16,7 @@
 // logits while pass 1 finishes and only then wait for pass 1's results.
 #include <cfloat>
 #include <climits>
+#include <cmath>
 #include <cstdio>
 
 #include "dard_internal.h"
@@ -114,15 +115,22 @@ __device__ __forceinline__ uint4 load_vec(const char* row, int e0, int c1) {
 
 // Folds VPT*W values (given by `val(v, e)`, element index `base + (v*256 + tid)*W + e`) into
 // the running accumulator: max/argmax first, then the exp-sum against the updated maximum.
-template <class T, int VPT, class ValFn>
-__device__ __forceinline__ void fold_round(Acc& acc, int base, ValFn val) {
+// With kTail, elements at or past `limit` (padding of the last round) count as -inf.
+template <class T, int VPT, bool kTail, class ValFn>
+__device__ __forceinline__ void fold_round(Acc& acc, int base, int limit, ValFn val) {
+  auto get = [&](int v, int e) {
+    const float x = val(v, e);
+    if (!kTail) return x;
+    const int i = base + (v * kScoreThreads + static_cast<int>(threadIdx.x)) * T::W + e;
+    return i < limit ? x : -INFINITY;
+  };
   float m = -INFINITY;
   int idx = INT_MAX;
 #pragma unroll
   for (int v = 0; v < VPT; ++v) {
 #pragma unroll
     for (int e = 0; e < T::W; ++e) {
-      const float x = val(v, e);
+      const float x = get(v, e);
       if (x > m) {
         m = x;
         idx = base + (v * kScoreThreads + static_cast<int>(threadIdx.x)) * T::W + e;
@@ -139,9 +147,15 @@ __device__ __forceinline__ void fold_round(Acc& acc, int base, ValFn val) {
 #pragma unroll
   for (int v = 0; v < VPT; ++v) {
 #pragma unroll
-    for (int e = 0; e < T::W; ++e) s += ex2_approx(fmaf(val(v, e), kLog2e, -mL));
+    for (int e = 0; e < T::W; ++e) s += ex2_approx(fmaf(get(v, e), kLog2e, -mL));
   }
   acc.s += s;
+}
+
+template <class T, int VPT, class ValFn>
+__device__ __forceinline__ void fold(Acc& acc, int base, int limit, ValFn val) {
+  if (base + kScoreThreads * VPT * T::W <= limit) fold_round<T, VPT, false>(acc, base, limit, val);
+  else fold_round<T, VPT, true>(acc, base, limit, val);
 }
 
 __device__ __forceinline__ Acc block_merge(Acc a, Acc* smem) {
@@ -268,7 +282,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
 #pragma unroll
     for (int v = 0; v < VPT; ++v)
       r[v] = load_vec<T>(rowp, base + (v * kScoreThreads + threadIdx.x) * T::W, c1);
-    fold_round<T, VPT>(acc, base, [&](int v, int e) { return T::get(r[v], e); });
+    fold<T, VPT>(acc, base, c1, [&](int v, int e) { return T::get(r[v], e); });
   }
   acc = block_merge(acc, s_acc);
   if (!publish_partial(p, row, split, acc, &s_last)) return;
@@ -283,7 +297,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
 template <class T, int VPT>
 __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_constant__ ScoreParams p) {
   __shared__ Acc s_acc[kWarps];
-  __shared__ double s_red[2][kWarps];
+  __shared__ double s_red[2][kWarps];  // only the first B/32 entries are used
   __shared__ int s_last;
   const int row = blockIdx.y, split = blockIdx.x;
   const int st = load_state(p, row, false);
@@ -311,33 +325,49 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   }
   grid_dep_wait();
 
-  // Eq. 5-6: w from the verification outcomes of this block (fp64, tree-summed).
+  // Eq. 5-6: w from the verification outcomes of this block (fp64, tree-summed terms
+  // lambda^|i-j| taken from the host-computed table).
   const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
   const int i = row - b0;
   double pp = 0.0, dd = 0.0;
-  for (int j = threadIdx.x; j < blen; j += kScoreThreads) {
-    const int f = __ldcg(p.pd_flag + b0 + j);
-    if (f != 0) {
-      const double kij = pow(static_cast<double>(p.lambda), static_cast<double>(abs(i - j)));
-      if (f == 1) pp += kij; else dd += kij;
+  if (blen > 32) {
+    for (int j = threadIdx.x; j < blen; j += kScoreThreads) {
+      const int f = __ldcg(p.pd_flag + b0 + j);
+      const double kij = p.lam_pow[abs(i - j)];
+      if (f == 1) pp += kij;
+      if (f == 2) dd += kij;
     }
-  }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    pp += __shfl_xor_sync(0xffffffffu, pp, off);
-    dd += __shfl_xor_sync(0xffffffffu, dd, off);
-  }
-  if ((threadIdx.x & 31) == 0) {
-    s_red[0][threadIdx.x >> 5] = pp;
-    s_red[1][threadIdx.x >> 5] = dd;
-  }
-  __syncthreads();
-  pp = 0.0;
-  dd = 0.0;
+    for (int off = 16; off > 0; off >>= 1) {
+      pp += __shfl_xor_sync(0xffffffffu, pp, off);
+      dd += __shfl_xor_sync(0xffffffffu, dd, off);
+    }
+    if ((threadIdx.x & 31) == 0) {
+      s_red[0][threadIdx.x >> 5] = pp;
+      s_red[1][threadIdx.x >> 5] = dd;
+    }
+    __syncthreads();
+    pp = 0.0;
+    dd = 0.0;
 #pragma unroll
-  for (int k = 0; k < kWarps; ++k) {
-    pp += s_red[0][k];
-    dd += s_red[1][k];
+    for (int k = 0; k < (DARD_MAX_BLOCK + 31) / 32; ++k) {
+      pp += s_red[0][k];
+      dd += s_red[1][k];
+    }
+  } else {
+    // one warp holds every term; every warp computes the same sum
+    const int lane = threadIdx.x & 31;
+    if (lane < blen) {
+      const int f = __ldcg(p.pd_flag + b0 + lane);
+      const double kij = p.lam_pow[abs(i - lane)];
+      pp = f == 1 ? kij : 0.0;
+      dd = f == 2 ? kij : 0.0;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      pp += __shfl_xor_sync(0xffffffffu, pp, off);
+      dd += __shfl_xor_sync(0xffffffffu, dd, off);
+    }
   }
   const double p0 = static_cast<double>(p.p0);
   const float w = static_cast<float>((pp + p0) / (pp + dd + p0));
@@ -348,7 +378,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
     return __fadd_rn(ls, __fmul_rn(w, __fsub_rn(lx, ls)));
   };
   Acc acc{-INFINITY, 0.f, INT_MAX};
-  fold_round<T, VPT>(acc, c0, [&](int v, int e) { return mix(rx[v], rs[v], e); });
+  fold<T, VPT>(acc, c0, c1, [&](int v, int e) { return mix(rx[v], rs[v], e); });
   for (int base = c0 + kScoreThreads * VPT * T::W; base < c1; base += kScoreThreads * VPT * T::W) {
 #pragma unroll
     for (int v = 0; v < VPT; ++v) {
@@ -356,7 +386,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
       rx[v] = load_vec<T>(xp, e0, c1);
       rs[v] = load_vec<T>(sp, e0, c1);
     }
-    fold_round<T, VPT>(acc, base, [&](int v, int e) { return mix(rx[v], rs[v], e); });
+    fold<T, VPT>(acc, base, c1, [&](int v, int e) { return mix(rx[v], rs[v], e); });
   }
   acc = block_merge(acc, s_acc);
   if (!publish_partial(p, row, split, acc, &s_last)) return;
@@ -424,6 +454,7 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
   }
   p.nsplit = nsplit;
   p.chunk = per_round * rounds;
+  for (int k = 0; k < DARD_MAX_BLOCK; ++k) p.lam_pow[k] = std::pow(static_cast<double>(p.lambda), k);
 
   char* ws = static_cast<char*>(a.workspace);
   auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };

@@ -21,7 +21,8 @@ def to_device(a: np.ndarray, dtype: str, device) -> torch.Tensor:
 
 
 class DeviceStep:
-    def __init__(self, wl: Workload, device="cuda", layers=None, attention=True, scoring=True):
+    def __init__(self, wl: Workload, device="cuda", layers=None, attention=True, scoring=True,
+                 logit_pitch: int | None = None):
         self.wl = wl
         self.device = torch.device(device)
         dt = wl.dtype
@@ -47,6 +48,14 @@ class DeviceStep:
         if scoring and wl.logits_s is not None:
             self.lx = to_device(wl.logits_x, dt, dev)
             self.ls = to_device(wl.logits_s, dt, dev)
+            if logit_pitch is not None and logit_pitch != wl.vocab:
+                # rows padded to `logit_pitch` elements; the padding holds a huge value that
+                # must never be read
+                for name in ("lx", "ls"):
+                    t = getattr(self, name)
+                    big = torch.full((t.shape[0], logit_pitch), 3.0e38, dtype=t.dtype, device=dev)
+                    big[:, :wl.vocab] = t
+                    setattr(self, name, big[:, :wl.vocab])
             nbytes = B.dard_score_workspace_size(self.rows, wl.vocab, len(wl.seqs))
             self.workspace = torch.zeros(max(nbytes, 16), dtype=torch.uint8, device=dev)
             r = max(self.rows, 1)

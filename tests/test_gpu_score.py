@@ -11,8 +11,8 @@ from . import parity as P
 pytestmark = pytest.mark.gpu
 
 
-def _run(wl, state_in=None, reps=1):
-    ds = DeviceStep(wl, attention=False)
+def _run(wl, state_in=None, reps=1, pitch=None):
+    ds = DeviceStep(wl, attention=False, logit_pitch=pitch)
     for _ in range(reps):
         ds.score(state_in=state_in)
     torch.cuda.synchronize()
@@ -57,7 +57,9 @@ def test_score_twice_in_a_row_same_result():
 def test_score_ragged_vocab_tails(vocab, dtype):
     specs = [dict(n_orig=40, block_start=8, block_len=24, fractions=(0.4, 0.3, 0.3))]
     wl = W.custom(specs, 1, 1, 64, dtype=dtype, vocab=vocab, seed=vocab, logit_std=2.0)
-    _check(wl, _run(wl)[1])
+    per16 = 8 if dtype == "bf16" else 4   # row pitch rounded up to 16 bytes
+    pitch = (vocab + per16 - 1) // per16 * per16
+    _check(wl, _run(wl, pitch=pitch + (per16 if vocab % 2 else 0))[1])
 
 
 def test_score_many_sequences_and_degenerate_blocks():
