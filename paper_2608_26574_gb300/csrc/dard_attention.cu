@@ -40,12 +40,15 @@ constexpr int kTcThreads = 192;
 constexpr uint32_t kTmemCols = 256;  // S/P buffers: columns [0,64), [64,128); O: [128, 128 + D)
 constexpr float kRescaleLog2 = 8.0f;
 
-// Per-CTA copy of the current block: states, confidences and the shadow maps.
-struct BlockInfo {
+// Per-CTA copy of the current block: states, confidences, the shadow maps, and the same
+// facts as bit words over block positions (word w = positions 32w .. 32w + 31).
+struct __align__(16) BlockInfo {
   int32_t st[DARD_MAX_BLOCK];
   float cf[DARD_MAX_BLOCK];
   int32_t shrow[DARD_MAX_BLOCK];  // block position -> shadow row index k, or -1
   int32_t shpos[DARD_MAX_BLOCK];  // shadow row index k -> block position, or -1 if invalid
+  uint32_t m_w[4], c_w[4], hs_w[4];  // state M, state C, has a (valid) shadow row
+  int32_t identity;                  // shpos[k] == k for every shadow row
 };
 
 // The query a row stands for: its copy (x or s), its state, c_{t-1}, block position.
@@ -74,27 +77,45 @@ __device__ __forceinline__ void decode_work(const AttnParams& p, int w, int& seq
   qt = local / p.hq;
 }
 
+// The block's per-position data as one thread fetches it from global memory (thread t:
+// block position t and shadow row t), so that the loads can be in flight early.
+struct BlockFetch {
+  int st;    // state of block position t, or -1
+  float cf;  // c_{t-1} of block position t
+  int pos;   // block position of shadow row t, or -1 past S
+};
+
+__device__ __forceinline__ BlockFetch fetch_block_info(const AttnParams& p, const SeqDesc& sd) {
+  const int t = threadIdx.x;
+  BlockFetch f{-1, 0.f, -1};
+  if (t < sd.blen) {
+    f.st = p.state[sd.blk_off + t];
+    f.cf = p.prev_conf[sd.blk_off + t];
+  }
+  if (t < sd.slen) f.pos = p.shadow_src[sd.sh_off + t] - sd.b0;
+  return f;
+}
+
 // Called by the 128 threads of warps 0-3. A repeated shadow position keeps its lowest
 // shadow row; the others, and positions outside the block, are flagged and never used.
-__device__ void load_block_info(const AttnParams& p, const SeqDesc& sd, BlockInfo& bi,
-                                bool report) {
+__device__ void publish_block_info(const AttnParams& p, const SeqDesc& sd, BlockInfo& bi,
+                                   const BlockFetch& f, bool report) {
   const int t = threadIdx.x;
   bi.shrow[t] = INT_MAX;
   bi.shpos[t] = -1;
   if (t < sd.blen) {
-    int s = p.state[sd.blk_off + t];
+    int s = f.st;
     if (s > 2) {
       if (report && p.status) atomicOr(p.status, DARD_STATUS_BAD_STATE);
       s = kStateM;
     }
     bi.st[t] = s;
-    bi.cf[t] = p.prev_conf[sd.blk_off + t];
+    bi.cf[t] = f.cf;
   }
-  int pos = -1;
-  if (t < sd.slen) pos = p.shadow_src[sd.sh_off + t] - sd.b0;
-  const bool in_block = pos >= 0 && pos < sd.blen;
+  const int pos = f.pos;
+  const bool in_block = t < sd.slen && pos >= 0 && pos < sd.blen;
   sm_bar_sync();
-  if (t < sd.slen && in_block) atomicMin(&bi.shrow[pos], t);
+  if (in_block) atomicMin(&bi.shrow[pos], t);
   sm_bar_sync();
   if (t < sd.slen) {
     const bool ok = in_block && bi.shrow[pos] == t;
@@ -103,7 +124,26 @@ __device__ void load_block_info(const AttnParams& p, const SeqDesc& sd, BlockInf
   }
   sm_bar_sync();
   if (bi.shrow[t] == INT_MAX) bi.shrow[t] = -1;
+  const int lane = t & 31, w = t >> 5;
+  const int s_t = t < sd.blen ? bi.st[t] : -1;
+  const uint32_t mw = __ballot_sync(0xffffffffu, s_t == kStateM);
+  const uint32_t cw = __ballot_sync(0xffffffffu, s_t == kStateC);
+  const uint32_t hw = __ballot_sync(0xffffffffu, t < sd.blen && bi.shrow[t] >= 0);
+  const uint32_t idw = __ballot_sync(0xffffffffu, t >= sd.slen || bi.shpos[t] == t);
+  if (lane == 0) {
+    bi.m_w[w] = mw;
+    bi.c_w[w] = cw;
+    bi.hs_w[w] = hw;
+  }
+  if (t == 0) bi.identity = 1;
   sm_bar_sync();
+  if (lane == 0 && idw != 0xffffffffu) bi.identity = 0;
+  sm_bar_sync();
+}
+
+__device__ __forceinline__ void load_block_info(const AttnParams& p, const SeqDesc& sd,
+                                                BlockInfo& bi, bool report) {
+  publish_block_info(p, sd, bi, fetch_block_info(p, sd), report);
 }
 
 __device__ __forceinline__ RowInfo row_info(const SeqDesc& sd, const BlockInfo& bi, int r) {
@@ -182,21 +222,62 @@ struct RowMasks {
   Bits128 see_s;
 };
 
+__device__ __forceinline__ Bits128 words128(const uint32_t (&w)[4]) {
+  return {static_cast<uint64_t>(w[0]) | (static_cast<uint64_t>(w[1]) << 32),
+          static_cast<uint64_t>(w[2]) | (static_cast<uint64_t>(w[3]) << 32)};
+}
+__device__ __forceinline__ Bits128 low_bits(int n) {  // bits [0, n), 0 <= n <= 128
+  Bits128 b;
+  b.lo = n >= 64 ? ~0ull : ((1ull << n) - 1);
+  b.hi = n >= 128 ? ~0ull : (n > 64 ? ((1ull << (n - 64)) - 1) : 0ull);
+  return b;
+}
+
+// The rule of takes_shadow() over all block positions at once, from the class words.
 __device__ RowMasks row_masks(const RowInfo& q, const BlockInfo& bi, const SeqDesc& sd) {
-  Bits128 ts{0, 0};  // takes_shadow for every block position
-  for (int j = 0; j < sd.blen; ++j)
-    if (takes_shadow(q, bi.st[j], bi.cf[j], j)) set_bit(ts, j);
-  RowMasks m{{0, 0}, {0, 0}};
-  for (int j = 0; j < sd.blen; ++j)
-    if (bi.shrow[j] >= 0 && get_bit(ts, j)) set_bit(m.hide_x, j);
-  for (int k = 0; k < sd.slen; ++k) {
-    const int j = bi.shpos[k];
-    if (j >= 0 && get_bit(ts, j)) set_bit(m.see_s, k);
+  const Bits128 mb = words128(bi.m_w), cb = words128(bi.c_w), hs = words128(bi.hs_w);
+  Bits128 ts{0, 0};
+  if (q.si == kStateU || (q.si == kStateM && q.qs)) {
+    ts = {mb.lo | cb.lo, mb.hi | cb.hi};
+  } else if (q.si == kStateC) {
+    // C keys with !(c_i <= c_j) come from s (Eq. 3); confidences read four at a time
+    Bits128 lower{0, 0};
+    const float4* cf4 = reinterpret_cast<const float4*>(bi.cf);
+    for (int j4 = 0; j4 < (sd.blen + 3) / 4; ++j4) {
+      const float4 c = cf4[j4];
+      const uint64_t nib = static_cast<uint64_t>(!(q.ci <= c.x)) |
+                           (static_cast<uint64_t>(!(q.ci <= c.y)) << 1) |
+                           (static_cast<uint64_t>(!(q.ci <= c.z)) << 2) |
+                           (static_cast<uint64_t>(!(q.ci <= c.w)) << 3);
+      const int j = 4 * j4;
+      if (j < 64) lower.lo |= nib << j; else lower.hi |= nib << (j - 64);
+    }
+    ts = {mb.lo | (cb.lo & lower.lo), mb.hi | (cb.hi & lower.hi)};
+  }
+  if (q.qs && q.i >= 0) set_bit(ts, q.i);  // a shadow query takes its own shadow key
+  RowMasks m;
+  m.hide_x = {ts.lo & hs.lo, ts.hi & hs.hi};
+  if (bi.identity) {
+    const Bits128 lim = low_bits(sd.slen);
+    m.see_s = {ts.lo & lim.lo, ts.hi & lim.hi};
+  } else {
+    m.see_s = {0, 0};
+    const int4* sp4 = reinterpret_cast<const int4*>(bi.shpos);
+    for (int k4 = 0; k4 < (sd.slen + 3) / 4; ++k4) {
+      const int4 jj = sp4[k4];
+      const int js[4] = {jj.x, jj.y, jj.z, jj.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int k = 4 * k4 + e;
+        if (k < sd.slen && js[e] >= 0 && get_bit(ts, js[e])) set_bit(m.see_s, k);
+      }
+    }
   }
   return m;
 }
 
 constexpr int kTN = 64;  // keys per tile of the tensor-core path
+constexpr int kL2Ahead = 8;  // K/V tiles prefetched into L2 ahead of the TMA loads
 
 __device__ __forceinline__ bool tile_needs_mask(const SeqDesc& sd, int kt0) {
   return (kt0 + kTN > sd.n_orig) ||
@@ -232,12 +313,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // behind the phase it waits for (the parity would alias otherwise). PV completion is
 // therefore tracked per S/P buffer (pv_done[b]: tiles b, b+2, ...), and the end of the
 // last PV by its own single-phase barrier o_full.
-struct __align__(8) TcCtl {
+struct __align__(16) TcCtl {
   uint64_t q_full, o_full;
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], p_full[2], pv_done[2];
   uint32_t tmem_base;
   int32_t abort;
   BlockInfo bi;
+  uint8_t store_row[kBM];  // epilogue: rows of this tile that are written
 };
 
 template <int D>
@@ -278,7 +360,27 @@ __global__ void __launch_bounds__(kTcThreads, 2)
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  if (threadIdx.x == 0) {
+  // The producer lane initialises the barriers and issues Q and the first two K/V tiles at
+  // once; the other threads touch the barriers only after the block-wide sync below.
+  const int row0 = sd.row_base;
+  auto load_kv = [&](int j, bool k_or_v) {
+    const int b = j & 1;
+    uint64_t* bar = k_or_v ? &ctl.k_full[b] : &ctl.v_full[b];
+    uint8_t* dst = (k_or_v ? sK : sV) + b * kKVBytes;
+    const void* map = k_or_v ? static_cast<const void*>(&tmk) : static_cast<const void*>(&tmv);
+    mbar_arrive_expect_tx(bar, kKVBytes);
+#pragma unroll
+    for (int s = 0; s < kSub; ++s)
+      tma_load_2d(dst + s * kKSub, map, bar, g * D + s * 64, row0 + j * kTN);
+  };
+  auto prefetch_kv = [&](int j) {
+#pragma unroll
+    for (int s = 0; s < kSub; ++s) {
+      tma_prefetch_l2_2d(&tmk, g * D + s * 64, row0 + j * kTN);
+      tma_prefetch_l2_2d(&tmv, g * D + s * 64, row0 + j * kTN);
+    }
+  };
+  if (warp == 4 && lane == 0) {
     mbar_init(&ctl.q_full, 1);
     mbar_init(&ctl.o_full, 1);
     for (int b = 0; b < 2; ++b) {
@@ -292,12 +394,25 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     }
     ctl.abort = 0;
     fence_barrier_init();
+    tma_prefetch_desc(&tmq);
+    tma_prefetch_desc(&tmk);
+    tma_prefetch_desc(&tmv);
+    mbar_arrive_expect_tx(&ctl.q_full, kQBytes);
+#pragma unroll
+    for (int s = 0; s < kSub; ++s)
+      tma_load_2d(sQ + s * kQSub, &tmq, &ctl.q_full, h * D + s * 64, row0 + q0);
+    for (int j = 0; j < 2 && j < n_kt; ++j) {
+      load_kv(j, true);
+      load_kv(j, false);
+    }
+    for (int j = 2; j < 2 + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
   }
-  if (warp == 4) {
+  if (warp == 5) {
     tmem_alloc<kTmemCols>(&ctl.tmem_base);
     tmem_relinquish();
   }
-  if (warp < 4) load_block_info(p, sd, ctl.bi, qt == 0 && h == 0);
+  BlockFetch bf{-1, 0.f, -1};
+  if (warp < 4) bf = fetch_block_info(p, sd);  // in flight across the block sync
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -307,30 +422,15 @@ __global__ void __launch_bounds__(kTcThreads, 2)
   if (warp == 4) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      tma_prefetch_desc(&tmq);
-      tma_prefetch_desc(&tmk);
-      tma_prefetch_desc(&tmv);
-      const int row0 = sd.row_base;
-      mbar_arrive_expect_tx(&ctl.q_full, kQBytes);
-#pragma unroll
-      for (int s = 0; s < kSub; ++s)
-        tma_load_2d(sQ + s * kQSub, &tmq, &ctl.q_full, h * D + s * 64, row0 + q0);
-      int last_k = -1, last_v = -1;
-      for (int j = 0; j < n_kt && !*abort_flag; ++j) {
+      int last_k = n_kt < 2 ? n_kt - 1 : 1, last_v = last_k;
+      for (int j = 2; j < n_kt && !*abort_flag; ++j) {
         const int b = j & 1;
-        if (j >= 2 && !mbar_wait(&ctl.k_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
-        mbar_arrive_expect_tx(&ctl.k_full[b], kKVBytes);
-#pragma unroll
-        for (int s = 0; s < kSub; ++s)
-          tma_load_2d(sK + b * kKVBytes + s * kKSub, &tmk, &ctl.k_full[b], g * D + s * 64,
-                      row0 + j * kTN);
+        if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
+        if (!mbar_wait(&ctl.k_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
+        load_kv(j, true);
         last_k = j;
-        if (j >= 2 && !mbar_wait(&ctl.v_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
-        mbar_arrive_expect_tx(&ctl.v_full[b], kKVBytes);
-#pragma unroll
-        for (int s = 0; s < kSub; ++s)
-          tma_load_2d(sV + b * kKVBytes + s * kKSub, &tmv, &ctl.v_full[b], g * D + s * 64,
-                      row0 + j * kTN);
+        if (!mbar_wait(&ctl.v_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
+        load_kv(j, false);
         last_v = j;
       }
       if (*abort_flag) {
@@ -387,6 +487,7 @@ __global__ void __launch_bounds__(kTcThreads, 2)
   } else {
     // ------------------------------------------------------------ softmax + epilogue
     const int t = threadIdx.x;
+    publish_block_info(p, sd, ctl.bi, bf, qt == 0 && h == 0);
     const RowInfo q = row_info(sd, ctl.bi, q0 + t);
     const RowMasks rm = row_masks(q, ctl.bi, sd);
     const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
@@ -411,17 +512,17 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         s[e] = __uint_as_float(r0[e]);
         s[32 + e] = __uint_as_float(r1[e]);
       }
-      float mt = -INFINITY;
       if (masked) {
 #pragma unroll
-        for (int k = 0; k < kTN; ++k) {
-          s[k] = ((vis >> k) & 1ull) ? s[k] : -INFINITY;
-          mt = fmaxf(mt, s[k]);
-        }
-      } else {
-#pragma unroll
-        for (int k = 0; k < kTN; ++k) mt = fmaxf(mt, s[k]);
+        for (int k = 0; k < kTN; ++k) s[k] = ((vis >> k) & 1ull) ? s[k] : -INFINITY;
       }
+      float mx[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = s[e];
+#pragma unroll
+      for (int k = 8; k < kTN; ++k) mx[k & 7] = fmaxf(mx[k & 7], s[k]);
+      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       // Raise the reference maximum on the first finite value, or when the tile maximum
       // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
       float m_new = m_run;
@@ -448,13 +549,15 @@ __global__ void __launch_bounds__(kTcThreads, 2)
       m_run = m_new;
       const float mL = (m_run == -INFINITY) ? 0.f : m_run * sl;
       uint32_t pk[32];
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
         const float a = ex2_approx(fmaf(s[2 * e], sl, -mL));
         const float c = ex2_approx(fmaf(s[2 * e + 1], sl, -mL));
-        l_run += a + c;
+        ls[e & 3] += a + c;
         pk[e] = pack_bf16x2(a, c);
       }
+      l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       tmem_st32(ctl.tmem_base + b * kTN + lane_off, pk);
       tmem_wait_st();
       tc_fence_before();
@@ -462,37 +565,53 @@ __global__ void __launch_bounds__(kTcThreads, 2)
       if (lane == 0) mbar_arrive(&ctl.p_full[b]);
     }
     if (ok) ok = mbar_wait(&ctl.o_full, 0);
-    if (!__all_sync(0xffffffffu, ok)) {
-      if (lane == 0) flag_timeout(p, ctl);
-    } else {
+    const bool wok = __all_sync(0xffffffffu, ok);
+    if (!wok && lane == 0) flag_timeout(p, ctl);
+    // O row / row sum -> bf16 into shared memory (the Q tile is no longer read once o_full
+    // has completed), 16-byte chunks XOR-swizzled by row; then the 128 threads store whole
+    // rows, coalesced. Every softmax warp reaches the named barrier on every path.
+    constexpr int kChunks = D / 8;  // 16-byte chunks per output row
+    const int r = q0 + t;
+    uint4* stage = reinterpret_cast<uint4*>(sQ);
+    if (wok) {
       tc_fence_after();
-      const int r = q0 + t;
-      const bool store = q.store && r < rows_seq;
       const float inv_l = 1.0f / l_run;
-      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o) +
-                           (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D;
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t rr[32];
         tmem_ld32(tO + lane_off + c * 32, rr);
         tmem_wait_ld();
-        if (store) {
-          uint32_t o2[16];
 #pragma unroll
-          for (int e = 0; e < 16; ++e)
-            o2[e] = pack_bf16x2(__uint_as_float(rr[2 * e]) * inv_l,
-                                __uint_as_float(rr[2 * e + 1]) * inv_l);
-          uint4* dst = reinterpret_cast<uint4*>(out + c * 32);
-#pragma unroll
-          for (int v = 0; v < 4; ++v)
-            dst[v] = make_uint4(o2[4 * v], o2[4 * v + 1], o2[4 * v + 2], o2[4 * v + 3]);
+        for (int v = 0; v < 4; ++v) {
+          uint4 u;
+          u.x = pack_bf16x2(__uint_as_float(rr[8 * v + 0]) * inv_l, __uint_as_float(rr[8 * v + 1]) * inv_l);
+          u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
+          u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
+          u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
+          const int chunk = c * 4 + v;
+          stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
+        }
+      }
+    }
+    ctl.store_row[t] = (wok && q.store && r < rows_seq) ? 1 : 0;
+    sm_bar_sync();
+    if (!*abort_flag) {
+      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o);
+#pragma unroll 4
+      for (int idx = t; idx < kBM * kChunks; idx += 128) {
+        const int row = idx / kChunks, chunk = idx % kChunks;
+        if (ctl.store_row[row]) {
+          const uint4 u = stage[row * kChunks + (chunk ^ (row & (kChunks - 1)))];
+          uint4* dst = reinterpret_cast<uint4*>(
+              out + (static_cast<size_t>(sd.row_base + q0 + row) * p.hq + h) * D);
+          dst[chunk] = u;
         }
       }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 4) {
+  if (warp == 5) {
     tc_fence_after();
     tmem_dealloc<kTmemCols>(ctl.tmem_base);
   }

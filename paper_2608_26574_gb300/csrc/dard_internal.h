@@ -59,9 +59,7 @@ struct ScoreParams {
   int32_t* counts;
   uint32_t* status;
   // workspace
-  float4* partial;     // [rows * nsplit] (max, sum, argmax bits, unused)
-  uint32_t* row_ctr;   // [rows]
-  uint32_t* seq_ctr;   // [num_seqs]
+  uint32_t* seq_ctr;   // [num_seqs] arrivals of the rows of a sequence (counts)
   uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 0 otherwise
   int64_t row_stride;
   int32_t vocab, rows, num_seqs, nsplit, chunk;
@@ -71,7 +69,7 @@ struct ScoreParams {
 };
 
 constexpr int kScoreThreads = 256;
-constexpr int kScoreMaxSplit = 64;
+constexpr int kScoreMaxSplit = 16;  // CTAs per row = thread-block cluster size
 
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs);
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,

@@ -9,13 +9,16 @@
 //   pass 2  rows in state M read both logit rows once, weight them by w from P and D of
 //           their own block and are decided.
 //
-// Both passes split every vocabulary row over `nsplit` CTAs (256 threads, 128-bit streaming
-// loads, warp-shuffle merge of (max, sum of exp, argmax)); the last CTA of a row, found with
-// an atomic counter, merges the per-split partials in a fixed order and writes the row's
-// outputs. Pass 2 is launched as a programmatic dependent of pass 1: its CTAs load their
-// logits while pass 1 finishes and only then wait for pass 1's results.
+// Both passes split every vocabulary row over the `nsplit` CTAs of one thread-block
+// cluster (256 threads each, 128-bit streaming loads, warp-shuffle merge of (max, sum of
+// exp, argmax)). Each CTA writes its partial into the shared memory of the cluster's first
+// CTA over DSMEM; after one cluster barrier that CTA merges the partials in split order
+// (deterministic) and writes the row's outputs. Pass 2 is launched as a programmatic
+// dependent of pass 1: its CTAs load their logits while pass 1 finishes and only then
+// wait for pass 1's results.
 #include <cfloat>
 #include <climits>
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 
@@ -188,28 +191,22 @@ __device__ __forceinline__ int load_state(const ScoreParams& p, int row, bool re
   return s;
 }
 
-// Publishes this CTA's partial; returns true (in every thread) for the row's last CTA.
-__device__ __forceinline__ bool publish_partial(const ScoreParams& p, int row, int split,
-                                                const Acc& a, int* s_flag) {
-  if (threadIdx.x == 0) {
-    p.partial[static_cast<size_t>(row) * p.nsplit + split] =
-        make_float4(a.m, a.s, __int_as_float(a.idx), 0.f);
-    __threadfence();
-    const uint32_t prev = atomicAdd(&p.row_ctr[row], 1u);
-    *s_flag = (prev == static_cast<uint32_t>(p.nsplit - 1));
-  }
-  __syncthreads();
-  return *s_flag != 0;
+// Sends this CTA's partial (warp 0 holds it) to slot `split` of the leader CTA (cluster
+// rank 0), then synchronises the cluster; afterwards the leader's slots are complete.
+__device__ __forceinline__ void cluster_publish(const Acc& a, int split, float4* slots) {
+  if (threadIdx.x == 0)
+    st_cluster_v4(map_shared_rank(smem_u32(&slots[split]), 0), a.m, a.s, __int_as_float(a.idx),
+                  0.f);
+  cluster_sync();
 }
 
-// Merges the row's partials in split order (warp 0); returns the row summary in lane 0.
-__device__ __forceinline__ Acc merge_partials(const ScoreParams& p, int row) {
-  __threadfence();
+// Merges the leader's slots in split order (warp 0); returns the row summary in lane 0.
+__device__ __forceinline__ Acc merge_slots(const float4* slots, int nsplit) {
   Acc a{-INFINITY, 0.f, INT_MAX};
   const int lane = threadIdx.x & 31;
-  for (int k = lane; k < p.nsplit; k += 32) {
-    const float4 v = __ldcg(&p.partial[static_cast<size_t>(row) * p.nsplit + k]);
-    a = acc_merge(a, Acc{v.x, v.y, __float_as_int(v.z)});
+  if (lane < nsplit) {
+    const float4 v = slots[lane];
+    a = Acc{v.x, v.y, __float_as_int(v.z)};
   }
   return warp_merge(a);
 }
@@ -226,7 +223,6 @@ __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const
   p.state_out[row] = static_cast<uint8_t>(ns);
   if (p.w_out) p.w_out[row] = w;
   if (!valid && p.status) atomicOr(p.status, DARD_STATUS_INVALID_ROW);
-  p.row_ctr[row] = 0u;  // leave the workspace zeroed for the next call
   return ns;
 }
 
@@ -266,10 +262,10 @@ template <class T, int VPT>
 __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_constant__ ScoreParams p) {
   grid_dep_launch();  // pass 2 may start loading its logits right away
   __shared__ Acc s_acc[kWarps];
-  __shared__ int s_last;
-  const int row = blockIdx.y, split = blockIdx.x;
+  __shared__ float4 s_slots[kScoreMaxSplit];
+  const int row = blockIdx.y, split = blockIdx.x;  // split = rank in the row's cluster
   const int st = load_state(p, row, split == 0);
-  if (st == kStateM) {
+  if (st == kStateM) {  // uniform over the cluster: no CTA of it reaches the barrier
     if (split == 0) p.pd_flag[row] = 0;
     return;
   }
@@ -285,9 +281,9 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
     fold<T, VPT>(acc, base, c1, [&](int v, int e) { return T::get(r[v], e); });
   }
   acc = block_merge(acc, s_acc);
-  if (!publish_partial(p, row, split, acc, &s_last)) return;
-  if (threadIdx.x >= 32) return;
-  const Acc a = merge_partials(p, row);
+  cluster_publish(acc, split, s_slots);
+  if (split != 0 || threadIdx.x >= 32) return;
+  const Acc a = merge_slots(s_slots, p.nsplit);
   if (threadIdx.x == 0) {
     const int ns = finalize_row(p, row, a, __int_as_float(0x7fc00000));
     p.pd_flag[row] = (st == kStateC) ? (ns == kStateU ? 1 : (ns == kStateM ? 2 : 0)) : 0;
@@ -297,8 +293,8 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
 template <class T, int VPT>
 __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_constant__ ScoreParams p) {
   __shared__ Acc s_acc[kWarps];
-  __shared__ double s_red[2][kWarps];  // only the first B/32 entries are used
-  __shared__ int s_last;
+  __shared__ float4 s_slots[kScoreMaxSplit];
+  __shared__ float s_w;
   const int row = blockIdx.y, split = blockIdx.x;
   const int st = load_state(p, row, false);
   const int seq = seq_of_row(p, row);
@@ -325,13 +321,14 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   }
   grid_dep_wait();
 
-  // Eq. 5-6: w from the verification outcomes of this block (fp64, tree-summed terms
-  // lambda^|i-j| taken from the host-computed table).
+  // Eq. 5-6: w from the verification outcomes of this block, computed by warp 0 alone in
+  // fp64 (the terms lambda^|i-j| come from the host table; the sum is a fixed tree) and
+  // broadcast through shared memory.
   const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
   const int i = row - b0;
-  double pp = 0.0, dd = 0.0;
-  if (blen > 32) {
-    for (int j = threadIdx.x; j < blen; j += kScoreThreads) {
+  if (threadIdx.x < 32) {
+    double pp = 0.0, dd = 0.0;
+    for (int j = threadIdx.x; j < blen; j += 32) {
       const int f = __ldcg(p.pd_flag + b0 + j);
       const double kij = p.lam_pow[abs(i - j)];
       if (f == 1) pp += kij;
@@ -342,35 +339,13 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
       pp += __shfl_xor_sync(0xffffffffu, pp, off);
       dd += __shfl_xor_sync(0xffffffffu, dd, off);
     }
-    if ((threadIdx.x & 31) == 0) {
-      s_red[0][threadIdx.x >> 5] = pp;
-      s_red[1][threadIdx.x >> 5] = dd;
-    }
-    __syncthreads();
-    pp = 0.0;
-    dd = 0.0;
-#pragma unroll
-    for (int k = 0; k < (DARD_MAX_BLOCK + 31) / 32; ++k) {
-      pp += s_red[0][k];
-      dd += s_red[1][k];
-    }
-  } else {
-    // one warp holds every term; every warp computes the same sum
-    const int lane = threadIdx.x & 31;
-    if (lane < blen) {
-      const int f = __ldcg(p.pd_flag + b0 + lane);
-      const double kij = p.lam_pow[abs(i - lane)];
-      pp = f == 1 ? kij : 0.0;
-      dd = f == 2 ? kij : 0.0;
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      pp += __shfl_xor_sync(0xffffffffu, pp, off);
-      dd += __shfl_xor_sync(0xffffffffu, dd, off);
+    if (threadIdx.x == 0) {
+      const double p0 = static_cast<double>(p.p0);
+      s_w = static_cast<float>((pp + p0) / (pp + dd + p0));
     }
   }
-  const double p0 = static_cast<double>(p.p0);
-  const float w = static_cast<float>((pp + p0) / (pp + dd + p0));
+  __syncthreads();
+  const float w = s_w;
 
   // Eq. 7 in fp32, one rounding per operation: mix = ls + w * (lx - ls).
   auto mix = [&](const uint4& vx, const uint4& vs, int e) {
@@ -389,9 +364,9 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
     fold<T, VPT>(acc, base, c1, [&](int v, int e) { return mix(rx[v], rs[v], e); });
   }
   acc = block_merge(acc, s_acc);
-  if (!publish_partial(p, row, split, acc, &s_last)) return;
-  if (threadIdx.x >= 32) return;
-  const Acc a = merge_partials(p, row);
+  cluster_publish(acc, split, s_slots);
+  if (split != 0 || threadIdx.x >= 32) return;
+  const Acc a = merge_slots(s_slots, p.nsplit);
   if (threadIdx.x == 0) finalize_row(p, row, a, w);
   if (p.counts != nullptr) {
     __syncwarp();
@@ -409,22 +384,41 @@ __global__ void zero_empty_counts(const __grid_constant__ ScoreParams p) {
     }
 }
 
+template <class F>
+cudaError_t allow_wide_clusters(F* kernel, std::atomic<uint64_t>& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (done.load(std::memory_order_acquire) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
+}
+
 template <class T, int VPT>
 cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
-  dim3 grid(p.nsplit, p.rows);
-  score_pass1<T, VPT><<<grid, kScoreThreads, 0, stream>>>(p);
-  cudaError_t e = cudaGetLastError();
+  static std::atomic<uint64_t> done1{0}, done2{0};
+  cudaError_t e = allow_wide_clusters(score_pass1<T, VPT>, done1);
+  if (e == cudaSuccess) e = allow_wide_clusters(score_pass2<T, VPT>, done2);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
+  cfg.gridDim = dim3(p.nsplit, p.rows);
   cfg.blockDim = dim3(kScoreThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.nsplit;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, score_pass1<T, VPT>, p);
+  if (e != cudaSuccess) return e;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, score_pass2<T, VPT>, p);
 }
 
@@ -432,39 +426,27 @@ cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
 
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs) {
   auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
-  return up(static_cast<size_t>(rows) * kScoreMaxSplit * sizeof(float4)) +
-         up(static_cast<size_t>(rows) * sizeof(uint32_t)) +
-         up(static_cast<size_t>(num_seqs) * sizeof(uint32_t)) + up(static_cast<size_t>(rows));
+  return up(static_cast<size_t>(num_seqs) * sizeof(uint32_t)) + up(static_cast<size_t>(rows));
 }
 
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
                          char* err, size_t err_len) {
   const bool bf16 = a.dtype == DARD_BF16;
   const int W = bf16 ? 8 : 4;
-  // Vectors per thread per round: 4, or 2 when the grid would otherwise leave SMs idle.
-  int vpt = 4;
-  int per_round = kScoreThreads * vpt * W;
-  if (static_cast<long long>(p.rows) * ((p.vocab + per_round - 1) / per_round) < 1216) vpt = 2;
-  per_round = kScoreThreads * vpt * W;
-  int nsplit = (p.vocab + per_round - 1) / per_round;
-  int rounds = 1;
-  if (nsplit > kScoreMaxSplit) {
-    rounds = (nsplit + kScoreMaxSplit - 1) / kScoreMaxSplit;
-    nsplit = (p.vocab + per_round * rounds - 1) / (per_round * rounds);
-  }
-  p.nsplit = nsplit;
+  // One round = 256 threads x 4 vectors; a row spreads over at most kScoreMaxSplit CTAs
+  // (one cluster), each taking `rounds` rounds.
+  const int per_round = kScoreThreads * 4 * W;
+  const int rounds_total = (p.vocab + per_round - 1) / per_round;
+  const int rounds = (rounds_total + kScoreMaxSplit - 1) / kScoreMaxSplit;
   p.chunk = per_round * rounds;
-  for (int k = 0; k < DARD_MAX_BLOCK; ++k) p.lam_pow[k] = std::pow(static_cast<double>(p.lambda), k);
+  p.nsplit = (p.vocab + p.chunk - 1) / p.chunk;
 
   char* ws = static_cast<char*>(a.workspace);
   auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
-  p.partial = reinterpret_cast<float4*>(ws);
-  ws += up(static_cast<size_t>(p.rows) * kScoreMaxSplit * sizeof(float4));
-  p.row_ctr = reinterpret_cast<uint32_t*>(ws);
-  ws += up(static_cast<size_t>(p.rows) * sizeof(uint32_t));
   p.seq_ctr = reinterpret_cast<uint32_t*>(ws);
   ws += up(static_cast<size_t>(p.num_seqs) * sizeof(uint32_t));
   p.pd_flag = reinterpret_cast<uint8_t*>(ws);
+  for (int k = 0; k < DARD_MAX_BLOCK; ++k) p.lam_pow[k] = std::pow(static_cast<double>(p.lambda), k);
 
   cudaError_t e = cudaSuccess;
   bool any_empty = false;
@@ -474,8 +456,7 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
     e = cudaGetLastError();
   }
   if (e == cudaSuccess && p.rows > 0) {
-    if (bf16) e = vpt == 4 ? launch_pair<Bf16, 4>(p, stream) : launch_pair<Bf16, 2>(p, stream);
-    else e = vpt == 4 ? launch_pair<F32, 4>(p, stream) : launch_pair<F32, 2>(p, stream);
+    e = bf16 ? launch_pair<Bf16, 4>(p, stream) : launch_pair<F32, 4>(p, stream);
   }
   if (e != cudaSuccess) {
     snprintf(err, err_len, "scoring launch failed: %s", cudaGetErrorString(e));
