@@ -129,7 +129,8 @@ dard_status dard_step_attention(const dard_attn_args* args, void* stream /* cuda
  *            mix = ls + w_i (lx - ls), each operation rounded to fp32              (Eq. 7)
  *            (c_i, x^_i) = (max softmax, argmax) of mix
  *   new state: c <= tau_c -> M, c <= tau_u -> C, else U                            (Eq. 8)
- * Argmax ties go to the lowest index. Softmax sums accumulate in fp32; w in fp64.
+ * Argmax ties go to the lowest index. Softmax sums and w accumulate in fp32 (the terms
+ * lambda^k as 2^(k log2 lambda)); w then enters Eq. 7 as an fp32 value.
  * Invalid rows (normaliser not finite or 0): conf 0, token -1, state M, status bit.
  * ------------------------------------------------------------------------------------- */
 typedef struct {
@@ -150,10 +151,10 @@ typedef struct {
   float* w_out;              /* optional device [rows] out: w for M rows, NaN otherwise    */
   int32_t* counts;           /* optional device [num_seqs * 3] out: M, C, U counts         */
   uint32_t* status;          /* optional device word, DARD_STATUS_* bits OR-ed in          */
-  void* workspace;           /* device scratch of dard_score_workspace_size() bytes, zeroed
-                                once by the caller after allocation; every call leaves it
-                                zeroed again. Calls that overlap on the GPU need separate
-                                workspaces.                                                */
+  void* workspace;           /* device scratch of dard_score_workspace_size() bytes (one
+                                byte per row: the promotion / demotion outcome of pass 1).
+                                No initial contents are needed. Calls that overlap on the
+                                GPU need separate workspaces.                              */
   size_t workspace_bytes;
 } dard_score_args;
 

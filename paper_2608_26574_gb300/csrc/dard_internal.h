@@ -59,12 +59,11 @@ struct ScoreParams {
   int32_t* counts;
   uint32_t* status;
   // workspace
-  uint32_t* seq_ctr;   // [num_seqs] arrivals of the rows of a sequence (counts)
   uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 0 otherwise
   int64_t row_stride;
   int32_t vocab, rows, num_seqs, nsplit, chunk;
   float tau_c, tau_u, lambda, p0;
-  double lam_pow[DARD_MAX_BLOCK];  // lambda^k, k = 0 .. DARD_MAX_BLOCK - 1 (Eq. 5 kernel)
+  float log2_lambda;  // lambda^k = 2^(k log2 lambda) (Eq. 5 kernel)
   int32_t blk_off[DARD_MAX_SEQS + 1];
 };
 

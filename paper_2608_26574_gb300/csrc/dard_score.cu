@@ -161,14 +161,39 @@ __device__ __forceinline__ void fold(Acc& acc, int base, int limit, ValFn val) {
   else fold_round<T, VPT, true>(acc, base, limit, val);
 }
 
+// Order-preserving map of non-NaN floats to unsigned integers (for redux.sync max).
+__device__ __forceinline__ uint32_t order_key(float x) {
+  const uint32_t b = __float_as_uint(x);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float from_key(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
+// Warp-wide merge: maximum and argmax by redux.sync, then one rescale per lane and a
+// shuffle tree for the sum (fixed order, so deterministic). m is never NaN (NaN values never
+// win a comparison); a NaN sum propagates.
+__device__ __forceinline__ Acc warp_merge_fast(const Acc& a) {
+  const uint32_t key = order_key(a.m);
+  const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+  const float mx = from_key(kmax);
+  const uint32_t cand = key == kmax ? static_cast<uint32_t>(a.idx) : 0xffffffffu;
+  const int idx = static_cast<int>(__reduce_min_sync(0xffffffffu, cand));
+  const float f = (a.m == -INFINITY) ? 0.f : ex2_approx((a.m - mx) * kLog2e);
+  float sum = a.s * f;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+  return {mx, sum, idx};
+}
+
 __device__ __forceinline__ Acc block_merge(Acc a, Acc* smem) {
-  a = warp_merge(a);
+  a = warp_merge_fast(a);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (lane == 0) smem[warp] = a;
   __syncthreads();
   if (warp == 0) {
     a = lane < kWarps ? smem[lane] : Acc{-INFINITY, 0.f, INT_MAX};
-    a = warp_merge(a);
+    a = warp_merge_fast(a);
   }
   return a;  // valid in warp 0
 }
@@ -226,36 +251,14 @@ __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const
   return ns;
 }
 
-// One arrival per row of a sequence in pass 2; the last one writes the M/C/U counts.
-__device__ __forceinline__ void arrive_counts(const ScoreParams& p, int seq) {
-  // called by a whole warp
-  const int lane = threadIdx.x & 31;
-  uint32_t last = 0;
-  const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
-  if (lane == 0) {
-    __threadfence();
-    last = atomicAdd(&p.seq_ctr[seq], 1u) == static_cast<uint32_t>(blen - 1);
-  }
-  last = __shfl_sync(0xffffffffu, last, 0);
-  if (!last) return;
-  __threadfence();
-  int cnt[3] = {0, 0, 0};
-  for (int j = lane; j < blen; j += 32) {
-    const int s = __ldcg(p.state_out + b0 + j);
-    cnt[0] += s == kStateM;
-    cnt[1] += s == kStateC;
-    cnt[2] += s == kStateU;
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1)
-#pragma unroll
-    for (int k = 0; k < 3; ++k) cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], off);
-  if (lane == 0) {
-    p.counts[seq * 3 + 0] = cnt[0];
-    p.counts[seq * 3 + 1] = cnt[1];
-    p.counts[seq * 3 + 2] = cnt[2];
-    p.seq_ctr[seq] = 0u;
-  }
+// M/C/U counts of every sequence: zeroed by one thread of pass 1, then every row adds its
+// final state in pass 2 (after the grid dependency, so the zeroing is visible).
+__device__ __forceinline__ void zero_counts(const ScoreParams& p) {
+  if (p.counts != nullptr && blockIdx.x == 0 && blockIdx.y == 0)
+    for (int k = threadIdx.x; k < 3 * p.num_seqs; k += blockDim.x) p.counts[k] = 0;
+}
+__device__ __forceinline__ void add_count(const ScoreParams& p, int seq, int state) {
+  if (p.counts != nullptr) atomicAdd(&p.counts[seq * 3 + state], 1);
 }
 
 template <class T, int VPT>
@@ -263,6 +266,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   grid_dep_launch();  // pass 2 may start loading its logits right away
   __shared__ Acc s_acc[kWarps];
   __shared__ float4 s_slots[kScoreMaxSplit];
+  zero_counts(p);
   const int row = blockIdx.y, split = blockIdx.x;  // split = rank in the row's cluster
   const int st = load_state(p, row, split == 0);
   if (st == kStateM) {  // uniform over the cluster: no CTA of it reaches the barrier
@@ -299,9 +303,9 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   const int st = load_state(p, row, false);
   const int seq = seq_of_row(p, row);
   if (st != kStateM) {
-    if (split == 0 && p.counts != nullptr && threadIdx.x < 32) {
+    if (split == 0 && p.counts != nullptr && threadIdx.x == 0) {
       grid_dep_wait();
-      arrive_counts(p, seq);
+      add_count(p, seq, __ldcg(p.state_out + row));
     }
     return;
   }
@@ -321,28 +325,24 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   }
   grid_dep_wait();
 
-  // Eq. 5-6: w from the verification outcomes of this block, computed by warp 0 alone in
-  // fp64 (the terms lambda^|i-j| come from the host table; the sum is a fixed tree) and
-  // broadcast through shared memory.
+  // Eq. 5-6: w from the verification outcomes of this block, computed by warp 0: each lane
+  // sums lambda^|i-j| = 2^(|i-j| log2 lambda) over its positions, then a shuffle tree.
   const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
   const int i = row - b0;
   if (threadIdx.x < 32) {
-    double pp = 0.0, dd = 0.0;
+    float pp = 0.f, dd = 0.f;
     for (int j = threadIdx.x; j < blen; j += 32) {
       const int f = __ldcg(p.pd_flag + b0 + j);
-      const double kij = p.lam_pow[abs(i - j)];
-      if (f == 1) pp += kij;
-      if (f == 2) dd += kij;
+      const float kij = ex2_approx(static_cast<float>(abs(i - j)) * p.log2_lambda);
+      pp += f == 1 ? kij : 0.f;
+      dd += f == 2 ? kij : 0.f;
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
       pp += __shfl_xor_sync(0xffffffffu, pp, off);
       dd += __shfl_xor_sync(0xffffffffu, dd, off);
     }
-    if (threadIdx.x == 0) {
-      const double p0 = static_cast<double>(p.p0);
-      s_w = static_cast<float>((pp + p0) / (pp + dd + p0));
-    }
+    if (threadIdx.x == 0) s_w = __fdiv_rn(pp + p.p0, pp + dd + p.p0);
   }
   __syncthreads();
   const float w = s_w;
@@ -367,21 +367,12 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   cluster_publish(acc, split, s_slots);
   if (split != 0 || threadIdx.x >= 32) return;
   const Acc a = merge_slots(s_slots, p.nsplit);
-  if (threadIdx.x == 0) finalize_row(p, row, a, w);
-  if (p.counts != nullptr) {
-    __syncwarp();
-    arrive_counts(p, seq);
-  }
+  if (threadIdx.x == 0) add_count(p, seq, finalize_row(p, row, a, w));
 }
 
-// Zeroes the counts of sequences without block rows (they get no arrivals).
-__global__ void zero_empty_counts(const __grid_constant__ ScoreParams p) {
-  for (int s = threadIdx.x; s < p.num_seqs; s += blockDim.x)
-    if (p.blk_off[s + 1] == p.blk_off[s]) {
-      p.counts[s * 3 + 0] = 0;
-      p.counts[s * 3 + 1] = 0;
-      p.counts[s * 3 + 2] = 0;
-    }
+// Zeroes the counts when there are no rows at all (no pass runs).
+__global__ void zero_all_counts(const __grid_constant__ ScoreParams p) {
+  for (int k = threadIdx.x; k < 3 * p.num_seqs; k += blockDim.x) p.counts[k] = 0;
 }
 
 template <class F>
@@ -425,8 +416,8 @@ cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
 }  // namespace
 
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs) {
-  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
-  return up(static_cast<size_t>(num_seqs) * sizeof(uint32_t)) + up(static_cast<size_t>(rows));
+  (void)num_seqs;
+  return (static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
 }
 
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
@@ -443,16 +434,12 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
 
   char* ws = static_cast<char*>(a.workspace);
   auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
-  p.seq_ctr = reinterpret_cast<uint32_t*>(ws);
-  ws += up(static_cast<size_t>(p.num_seqs) * sizeof(uint32_t));
   p.pd_flag = reinterpret_cast<uint8_t*>(ws);
-  for (int k = 0; k < DARD_MAX_BLOCK; ++k) p.lam_pow[k] = std::pow(static_cast<double>(p.lambda), k);
+  p.log2_lambda = static_cast<float>(std::log2(static_cast<double>(p.lambda)));
 
   cudaError_t e = cudaSuccess;
-  bool any_empty = false;
-  for (int s = 0; s < p.num_seqs; ++s) any_empty |= p.blk_off[s + 1] == p.blk_off[s];
-  if (p.counts != nullptr && any_empty) {
-    zero_empty_counts<<<1, 256, 0, stream>>>(p);
+  if (p.counts != nullptr && p.rows == 0) {
+    zero_all_counts<<<1, 256, 0, stream>>>(p);
     e = cudaGetLastError();
   }
   if (e == cudaSuccess && p.rows > 0) {

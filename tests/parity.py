@@ -8,6 +8,7 @@ import oracle as orc
 BORDER = 1e-5      # |c - tau| below this: the transition may legitimately go either way
 NEAR_TIE = 1e-3    # top-2 logit gap below this: the argmax may legitimately differ
 CONF_TOL = 1e-4    # confidences, fp32 accumulation
+W_REL = 4e-6       # guidance weight: fp32 sum of at most 128 terms against fp64
 ATT_MAX_ABS = 2e-2
 ATT_MEAN_ABS = 1e-2
 
@@ -82,7 +83,7 @@ def compare_scores(wl, conf, token, state_out, w_out=None, counts=None):
     gap under NEAR_TIE. Returns a report dict; raises AssertionError on any mismatch."""
     offs = wl.block_offsets()
     taus = (f32(wl.tau_c), f32(wl.tau_u))
-    rep = {"rows": 0, "borderline": 0, "near_tie": 0, "max_conf_err": 0.0, "max_w_ulps": 0.0}
+    rep = {"rows": 0, "borderline": 0, "near_tie": 0, "max_conf_err": 0.0, "max_w_rel": 0.0}
     for si, (s, res) in enumerate(zip(wl.seqs, oracle_scores(wl))):
         a, b = offs[si], offs[si + 1]
         st = np.where(s.state > 2, 0, s.state)
@@ -100,9 +101,11 @@ def compare_scores(wl, conf, token, state_out, w_out=None, counts=None):
             if st[i] == 0:
                 row = orc.mix_logits(wl.logits_x[r], wl.logits_s[r], res.w[i])
                 if w_out is not None:
-                    ulps = abs(float(w_out[r]) - float(res.w[i])) / float(np.spacing(np.float32(res.w[i])))
-                    rep["max_w_ulps"] = max(rep["max_w_ulps"], ulps)
-                    assert ulps <= 2, (si, i, w_out[r], res.w[i])
+                    # the kernel sums the Eq. 5 terms in fp32 (2^(k log2 lambda) on the SFU),
+                    # the oracle in fp64: relative agreement to W_REL
+                    rel = abs(float(w_out[r]) - float(res.w[i])) / float(res.w[i])
+                    rep["max_w_rel"] = max(rep["max_w_rel"], rel)
+                    assert rel <= W_REL, (si, i, w_out[r], res.w[i])
             else:
                 row = wl.logits_s[r]
                 if w_out is not None:
