@@ -8,11 +8,17 @@
 // so the mask is evaluated only on the (at most three) tiles that contain block keys,
 // shadow keys or the ragged end of the sequence.
 //
-// bf16 path (attn_tc): one CTA = 128 query rows of one (sequence, head); 6 warps:
+// bf16 path (attn_tc): one CTA per SM = 128 query rows of one (sequence, head); 6 warps:
 //   warps 0-3  softmax and epilogue, thread t owns query row t (= TMEM lane t);
-//   warp 4     TMA producer (Q once, then K and V tiles of 128 keys) and TMEM allocator;
-//   warp 5     tcgen05 MMA issuer: S = Q K^T into TMEM, then O += P V with P (bf16) read
-//              from TMEM where the softmax warps wrote it over S.
+//   warp 4     TMA producer: Q once, then K and V tiles of 64 keys through 4 stages each,
+//              with L2 prefetches a few tiles further ahead;
+//   warp 5     TMEM allocator and PV issuer: O += P_j V_j with P_j (bf16) read from TMEM
+//              where the softmax warps wrote it over S_j;
+//   warp 6     S issuer: S_j = Q K_j^T (tcgen05, Q from TMEM, K from shared memory) into a
+//              ring of four 64-column TMEM buffers. With its own issuing thread S runs up
+//              to four tiles ahead of the softmax and is never held up behind a PV wait.
+// The softmax threads write their query rows into TMEM (bf16 pairs, the A-operand layout)
+// at the start, so shared-memory bandwidth goes to K and V only.
 // The online softmax keeps a per-row running maximum and rescales O in TMEM only when the
 // maximum grows by more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
 // fp32 path (attn_simt): CUDA-core kernel, one warp per query row, same mask logic.
@@ -36,8 +42,9 @@ namespace dard {
 namespace {
 
 constexpr int kBM = 128;  // query rows per CTA
-constexpr int kTcThreads = 192;
-constexpr uint32_t kTmemCols = 256;  // S/P buffers: columns [0,64), [64,128); O: [128, 128 + D)
+constexpr int kTcThreads = 352;  // 8 softmax warps, producer, PV issuer, S issuer
+constexpr uint32_t kTmemCols = 512;  // S/P ring: 2 x 128 columns [0, 256); O: [256, 256 + D);
+                                     // Q (bf16 pairs): [384, 384 + D / 2)
 constexpr float kRescaleLog2 = 8.0f;
 
 // Per-CTA copy of the current block: states, confidences, the shadow maps, and the same
@@ -276,8 +283,8 @@ __device__ RowMasks row_masks(const RowInfo& q, const BlockInfo& bi, const SeqDe
   return m;
 }
 
-constexpr int kTN = 64;  // keys per tile of the tensor-core path
-constexpr int kL2Ahead = 8;  // K/V tiles prefetched into L2 ahead of the TMA loads
+constexpr int kTN = 128;  // keys per tile of the tensor-core path
+constexpr int kL2Ahead = 4;  // K/V tiles prefetched into L2 ahead of the TMA loads
 
 __device__ __forceinline__ bool tile_needs_mask(const SeqDesc& sd, int kt0) {
   return (kt0 + kTN > sd.n_orig) ||
@@ -285,16 +292,16 @@ __device__ __forceinline__ bool tile_needs_mask(const SeqDesc& sd, int kt0) {
 }
 
 // Visibility of keys [kt0, kt0 + 64) for one row (bit t = key kt0 + t).
-__device__ __forceinline__ uint64_t tile_visibility(const SeqDesc& sd, int kt0, const RowMasks& m) {
+__device__ __forceinline__ uint64_t vis64(const SeqDesc& sd, int kt0, const RowMasks& m) {
   uint64_t vis = ~0ull;
-  const int lo = max(kt0, sd.b0), hi = min(kt0 + kTN, sd.b0 + sd.blen);
+  const int lo = max(kt0, sd.b0), hi = min(kt0 + 64, sd.b0 + sd.blen);
   if (lo < hi) {
     const int len = hi - lo;
     uint64_t h = bits_window(m.hide_x, lo - sd.b0);
     if (len < 64) h &= (1ull << len) - 1;
     vis &= ~(h << (lo - kt0));
   }
-  if (kt0 + kTN > sd.n_orig) {
+  if (kt0 + 64 > sd.n_orig) {
     const int s_lo = max(kt0, sd.n_orig);
     const int off = s_lo - kt0;  // 0..63
     const uint64_t keep = off == 0 ? 0ull : ((1ull << off) - 1);
@@ -309,24 +316,40 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
-// Every barrier below completes one phase per use; a waiter is never more than one phase
-// behind the phase it waits for (the parity would alias otherwise). PV completion is
-// therefore tracked per S/P buffer (pv_done[b]: tiles b, b+2, ...), and the end of the
-// last PV by its own single-phase barrier o_full.
+constexpr int kNS = 2;   // S buffers in TMEM (a ring of 128-column buffers)
+constexpr int kNKV = 3;  // TMA stages for K and for V
+constexpr int kSoftmaxWarps = 8;  // two warps per query row, 64 key columns each
+
+// Named barriers: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = all softmax warps,
+// 3 + q = the two warps (q and q + 4) that share TMEM lane quarter q.
+__device__ __forceinline__ void softmax_bar_sync() {
+  asm volatile("bar.sync 2, 256;" ::: "memory");
+}
+__device__ __forceinline__ void pair_bar_sync(int quarter) {
+  asm volatile("bar.sync %0, 64;" ::"r"(3 + quarter) : "memory");
+}
+
+// Every barrier completes one phase per use of its ring slot; tile j uses slot j % ring
+// and waits for parity (j / ring) & 1. A waiter is never more than one phase behind the
+// phase it waits for (the parity would alias otherwise): each wait for use u of a slot is
+// preceded, in the same thread or through a chain of waits, by the completion of use u - 1.
 struct __align__(16) TcCtl {
-  uint64_t q_full, o_full;
-  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], p_full[2], pv_done[2];
+  uint64_t q_full, o_full, p_full, pv_done;
+  uint64_t k_full[kNKV], k_empty[kNKV], v_full[kNKV], v_empty[kNKV];
+  uint64_t s_full[kNS], s_free[kNS];
   uint32_t tmem_base;
   int32_t abort;
   BlockInfo bi;
+  float red_max[2][2][kBM];  // per tile (double-buffered by tile parity): the two column
+                             // halves' row maxima
+  float red_sum[2][kBM];   // at the end: the two halves' row sums
   uint8_t store_row[kBM];  // epilogue: rows of this tile that are written
 };
 
 template <int D>
 constexpr size_t tc_smem_bytes() {
-  // alignment slack + Q (128 rows) + two stages each of K and V (64 rows) + control
-  return 1024 + static_cast<size_t>(kBM) * D * 2 + 4 * static_cast<size_t>(kTN) * D * 2 +
-         sizeof(TcCtl);
+  // alignment slack + kNKV stages each of K and V (128 rows) + control
+  return 1024 + 2 * kNKV * static_cast<size_t>(kTN) * D * 2 + sizeof(TcCtl);
 }
 
 __device__ __forceinline__ void flag_timeout(const AttnParams& p, TcCtl& ctl) {
@@ -335,21 +358,19 @@ __device__ __forceinline__ void flag_timeout(const AttnParams& p, TcCtl& ctl) {
 }
 
 template <int D>
-__global__ void __launch_bounds__(kTcThreads, 2)
-    attn_tc(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmq,
-            const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv) {
+__global__ void __launch_bounds__(kTcThreads, 1)
+    attn_tc(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmk,
+            const __grid_constant__ CUtensorMap tmv) {
   constexpr int kSub = D / 64;                 // 128-byte (64 x bf16) column blocks
-  constexpr uint32_t kQSub = kBM * 128;        // one 128-row x 128-byte swizzled block
-  constexpr uint32_t kKSub = kTN * 128;        // one 64-row x 128-byte swizzled block
-  constexpr uint32_t kQBytes = kSub * kQSub;
-  constexpr uint32_t kKVBytes = kSub * kKSub;  // one K (or V) tile of 64 keys
+  constexpr uint32_t kKSub = kTN * 128;        // one 128-row x 128-byte swizzled block
+  constexpr uint32_t kKVBytes = kSub * kKSub;  // one K (or V) tile of 128 keys
+  constexpr int kWProd = kSoftmaxWarps, kWPV = kSoftmaxWarps + 1, kWS = kSoftmaxWarps + 2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sQ = base;
-  uint8_t* sK = sQ + kQBytes;        // stages at sK, sK + kKVBytes
-  uint8_t* sV = sK + 2 * kKVBytes;   // stages at sV, sV + kKVBytes
-  TcCtl& ctl = *reinterpret_cast<TcCtl*>(sV + 2 * kKVBytes);
+  uint8_t* sK = base;                  // kNKV stages
+  uint8_t* sV = sK + kNKV * kKVBytes;  // kNKV stages
+  TcCtl& ctl = *reinterpret_cast<TcCtl*>(sV + kNKV * kKVBytes);
 
   int seq, qt, h;
   decode_work(p, blockIdx.x, seq, qt, h);
@@ -360,11 +381,11 @@ __global__ void __launch_bounds__(kTcThreads, 2)
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // The producer lane initialises the barriers and issues Q and the first two K/V tiles at
+  // The producer lane initialises the barriers and issues the first kNKV K/V tiles at
   // once; the other threads touch the barriers only after the block-wide sync below.
   const int row0 = sd.row_base;
   auto load_kv = [&](int j, bool k_or_v) {
-    const int b = j & 1;
+    const int b = j % kNKV;
     uint64_t* bar = k_or_v ? &ctl.k_full[b] : &ctl.v_full[b];
     uint8_t* dst = (k_or_v ? sK : sV) + b * kKVBytes;
     const void* map = k_or_v ? static_cast<const void*>(&tmk) : static_cast<const void*>(&tmv);
@@ -380,206 +401,283 @@ __global__ void __launch_bounds__(kTcThreads, 2)
       tma_prefetch_l2_2d(&tmv, g * D + s * 64, row0 + j * kTN);
     }
   };
-  if (warp == 4 && lane == 0) {
-    mbar_init(&ctl.q_full, 1);
+  if (warp == kWProd && lane == 0) {
+    mbar_init(&ctl.q_full, kSoftmaxWarps);  // each softmax warp writes half of its Q rows
     mbar_init(&ctl.o_full, 1);
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&ctl.pv_done[b], 1);
+    mbar_init(&ctl.p_full, kSoftmaxWarps);
+    mbar_init(&ctl.pv_done, 1);
+    for (int b = 0; b < kNKV; ++b) {
       mbar_init(&ctl.k_full[b], 1);
       mbar_init(&ctl.k_empty[b], 1);
       mbar_init(&ctl.v_full[b], 1);
       mbar_init(&ctl.v_empty[b], 1);
+    }
+    for (int b = 0; b < kNS; ++b) {
       mbar_init(&ctl.s_full[b], 1);
-      mbar_init(&ctl.p_full[b], 4);
+      mbar_init(&ctl.s_free[b], kSoftmaxWarps);
     }
     ctl.abort = 0;
     fence_barrier_init();
-    tma_prefetch_desc(&tmq);
     tma_prefetch_desc(&tmk);
     tma_prefetch_desc(&tmv);
-    mbar_arrive_expect_tx(&ctl.q_full, kQBytes);
-#pragma unroll
-    for (int s = 0; s < kSub; ++s)
-      tma_load_2d(sQ + s * kQSub, &tmq, &ctl.q_full, h * D + s * 64, row0 + q0);
-    for (int j = 0; j < 2 && j < n_kt; ++j) {
+    for (int j = 0; j < kNKV && j < n_kt; ++j) {
       load_kv(j, true);
       load_kv(j, false);
     }
-    for (int j = 2; j < 2 + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
+    for (int j = kNKV; j < kNKV + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
   }
-  if (warp == 5) {
+  if (warp == kWPV) {
     tmem_alloc<kTmemCols>(&ctl.tmem_base);
     tmem_relinquish();
   }
+  // Softmax warp w: rows 32 (w % 4) .. + 31 (TMEM lane quarter), key columns 64 (w / 4) ..
+  const int quarter = warp & 3, half = warp >> 2;
+  const int t = quarter * 32 + lane;  // this thread's query row within the tile
   BlockFetch bf{-1, 0.f, -1};
-  if (warp < 4) bf = fetch_block_info(p, sd);  // in flight across the block sync
+  uint4 qhalf[D / 16];  // half of this thread's query row (bf16)
+  if (warp < kSoftmaxWarps) {
+    if (half == 0) bf = fetch_block_info(p, sd);  // in flight across the block sync
+    const int r = row0 + q0 + t;
+    const uint4* src = reinterpret_cast<const uint4*>(
+        static_cast<const __nv_bfloat16*>(p.q) + (static_cast<size_t>(r) * p.hq + h) * D +
+        half * (D / 2));
+#pragma unroll
+    for (int c = 0; c < D / 16; ++c)
+      qhalf[c] = r < p.total_rows ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tO = ctl.tmem_base + 128;
+  // TMEM columns: S ring [0, 256), O [256, 256 + D), P [384, 448), Q [448, 448 + D / 2)
+  const uint32_t tO = ctl.tmem_base + kNS * kTN;
+  const uint32_t tP = ctl.tmem_base + 384;
+  const uint32_t tQ = ctl.tmem_base + 448;
   volatile int32_t* abort_flag = &ctl.abort;
 
-  if (warp == 4) {
+  if (warp == kWProd) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      int last_k = n_kt < 2 ? n_kt - 1 : 1, last_v = last_k;
-      for (int j = 2; j < n_kt && !*abort_flag; ++j) {
-        const int b = j & 1;
+      int last_k = min(n_kt, kNKV) - 1, last_v = last_k;
+      for (int j = kNKV; j < n_kt && !*abort_flag; ++j) {
+        const int b = j % kNKV, ph = ((j - kNKV) / kNKV) & 1;
         if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
-        if (!mbar_wait(&ctl.k_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
+        if (!mbar_wait(&ctl.k_empty[b], ph)) { flag_timeout(p, ctl); break; }
         load_kv(j, true);
         last_k = j;
-        if (!mbar_wait(&ctl.v_empty[b], ((j - 2) >> 1) & 1)) { flag_timeout(p, ctl); break; }
+        if (!mbar_wait(&ctl.v_empty[b], ph)) { flag_timeout(p, ctl); break; }
         load_kv(j, false);
         last_v = j;
       }
       if (*abort_flag) {
         // let the copies already in flight land before shared memory is released
-        if (last_k >= 0) mbar_wait(&ctl.k_full[last_k & 1], (last_k >> 1) & 1);
-        if (last_v >= 0) mbar_wait(&ctl.v_full[last_v & 1], (last_v >> 1) & 1);
+        if (last_k >= 0) mbar_wait(&ctl.k_full[last_k % kNKV], (last_k / kNKV) & 1);
+        if (last_v >= 0) mbar_wait(&ctl.v_full[last_v % kNKV], (last_v / kNKV) & 1);
       }
     }
-  } else if (warp == 5) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == kWS) {
+    // ------------------------------------------------------------ S issuer
+    // S_t = Q K_t^T (Q from TMEM, K from shared memory) into ring buffer t % kNS as soon as
+    // K_t has landed and the softmax has read S_{t - kNS} out of that buffer.
     if (lane == 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
-      constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
-      const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK), av = smem_u32(sV);
-      auto issue_s = [&](int t) -> bool {  // S_t = Q K_t^T into S buffer t & 1
-        const int b = t & 1;
-        if (!mbar_wait(&ctl.k_full[b], (t >> 1) & 1)) return false;
-        tc_fence_after();
-        const uint32_t kb = ak + b * kKVBytes;
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t qo = (ks >> 2) * kQSub + (ks & 3) * 32;
-          const uint32_t ko = (ks >> 2) * kKSub + (ks & 3) * 32;
-          mma_ss(ctl.tmem_base + b * kTN, smem_desc_sw128(aq + qo, 16, 1024),
-                 smem_desc_sw128(kb + ko, 16, 1024), kIdS, ks > 0);
-        }
-        mma_commit(&ctl.s_full[b]);
-        mma_commit(&ctl.k_empty[b]);
-        return true;
-      };
+      const uint32_t ak = smem_u32(sK);
       bool ok = mbar_wait(&ctl.q_full, 0);
-      if (ok) ok = issue_s(0);
-      if (ok && n_kt > 1) ok = issue_s(1);
-      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
-        const int b = j & 1;
-        ok = mbar_wait(&ctl.p_full[b], (j >> 1) & 1) && mbar_wait(&ctl.v_full[b], (j >> 1) & 1);
+      for (int t2 = 0; t2 < n_kt && ok && !*abort_flag; ++t2) {
+        const int kb = t2 % kNKV, sb = t2 % kNS;
+        if (t2 >= kNS) ok = mbar_wait(&ctl.s_free[sb], ((t2 - kNS) / kNS) & 1);
+        ok = ok && mbar_wait(&ctl.k_full[kb], (t2 / kNKV) & 1);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t vb = av + b * kKVBytes;
+        const uint32_t kaddr = ak + kb * kKVBytes;
+        const uint32_t dst = ctl.tmem_base + sb * kTN;
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t ko = (ks >> 2) * kKSub + (ks & 3) * 32;
+          mma_ts(dst, tQ + ks * 8, smem_desc_sw128(kaddr + ko, 16, 1024), kIdS, ks > 0);
+        }
+        mma_commit(&ctl.s_full[sb]);
+        mma_commit(&ctl.k_empty[kb]);
+      }
+      if (!ok) flag_timeout(p, ctl);
+    }
+  } else if (warp == kWPV) {
+    // ------------------------------------------------------------ PV issuer
+    // O += P_j V_j as soon as the softmax has written P_j and V_j has landed.
+    if (lane == 0) {
+      constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
+      const uint32_t av = smem_u32(sV);
+      bool ok = true;
+      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
+        const int vb = j % kNKV;
+        ok = mbar_wait(&ctl.p_full, j & 1) && mbar_wait(&ctl.v_full[vb], (j / kNKV) & 1);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t vaddr = av + vb * kKVBytes;
 #pragma unroll
         for (int ks = 0; ks < kTN / 16; ++ks)
-          mma_ts(tO, ctl.tmem_base + b * kTN + ks * 8,
-                 smem_desc_sw128(vb + ks * 2048, kKSub, 1024), kIdO, (j > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&ctl.pv_done[b]);
-        mma_commit(&ctl.v_empty[b]);
+          mma_ts(tO, tP + ks * 8, smem_desc_sw128(vaddr + ks * 2048, kKSub, 1024), kIdO,
+                 (j > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&ctl.pv_done);
+        mma_commit(&ctl.v_empty[vb]);
         if (j == n_kt - 1) mma_commit(&ctl.o_full);
-        if (j + 2 < n_kt) {
-          // S buffer b is free once PV_j has read P_j out of it
-          ok = mbar_wait(&ctl.pv_done[b], (j >> 1) & 1) && issue_s(j + 2);
-        }
       }
       if (!ok) flag_timeout(p, ctl);
     }
   } else {
     // ------------------------------------------------------------ softmax + epilogue
-    const int t = threadIdx.x;
-    publish_block_info(p, sd, ctl.bi, bf, qt == 0 && h == 0);
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    {  // this warp's half of the query rows into TMEM (bf16 pairs, the A-operand layout)
+#pragma unroll
+      for (int c = 0; c < D / 128; ++c) {
+        uint32_t w[32];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          w[4 * e + 0] = qhalf[8 * c + e].x;
+          w[4 * e + 1] = qhalf[8 * c + e].y;
+          w[4 * e + 2] = qhalf[8 * c + e].z;
+          w[4 * e + 3] = qhalf[8 * c + e].w;
+        }
+        tmem_st32(tQ + lane_off + half * (D / 4) + 32 * c, w);
+      }
+      if (D == 64) {  // 16 columns per half
+        uint32_t w[16];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          w[4 * e + 0] = qhalf[e].x;
+          w[4 * e + 1] = qhalf[e].y;
+          w[4 * e + 2] = qhalf[e].z;
+          w[4 * e + 3] = qhalf[e].w;
+        }
+        tmem_st16(tQ + lane_off + half * 16, w);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.q_full);
+    }
+    if (half == 0) publish_block_info(p, sd, ctl.bi, bf, qt == 0 && h == 0);
+    softmax_bar_sync();
     const RowInfo q = row_info(sd, ctl.bi, q0 + t);
     const RowMasks rm = row_masks(q, ctl.bi, sd);
-    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
     const float sl = p.scale_log2;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < n_kt; ++j) {
-      const int b = j & 1;
-      const int kt0 = j * kTN;
-      const bool masked = tile_needs_mask(sd, kt0);
-      const uint64_t vis = masked ? tile_visibility(sd, kt0, rm) : ~0ull;
-      ok = !*abort_flag && mbar_wait(&ctl.s_full[b], (j >> 1) & 1);
+      const int b = j % kNS;
+      const int kt0 = j * kTN + half * 64;  // this warp's 64 keys
+      const bool masked = tile_needs_mask(sd, j * kTN);
+      const uint64_t vis = masked ? vis64(sd, kt0, rm) : ~0ull;
+      ok = !*abort_flag && mbar_wait(&ctl.s_full[b], (j / kNS) & 1);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
-      uint32_t r0[32], r1[32];
-      tmem_ld32(ctl.tmem_base + b * kTN + lane_off, r0);
-      tmem_ld32(ctl.tmem_base + b * kTN + 32 + lane_off, r1);
-      tmem_wait_ld();
-      float s[kTN];
+      float s[64];
+      {
+        uint32_t r0[32], r1[32];
+        tmem_ld32(ctl.tmem_base + b * kTN + 64 * half + lane_off, r0);
+        tmem_ld32(ctl.tmem_base + b * kTN + 64 * half + 32 + lane_off, r1);
+        tmem_wait_ld();
 #pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        s[e] = __uint_as_float(r0[e]);
-        s[32 + e] = __uint_as_float(r1[e]);
+        for (int e = 0; e < 32; ++e) {
+          s[e] = __uint_as_float(r0[e]);
+          s[32 + e] = __uint_as_float(r1[e]);
+        }
       }
+      // S_j is in registers: the S issuer may reuse its buffer
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.s_free[b]);
       if (masked) {
 #pragma unroll
-        for (int k = 0; k < kTN; ++k) s[k] = ((vis >> k) & 1ull) ? s[k] : -INFINITY;
+        for (int k = 0; k < 64; ++k) s[k] = ((vis >> k) & 1ull) ? s[k] : -INFINITY;
       }
       float mx[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) mx[e] = s[e];
+      for (int e = 0; e < 8; ++e) mx[e] = fmax3(s[e], s[8 + e], s[16 + e]);
 #pragma unroll
-      for (int k = 8; k < kTN; ++k) mx[k & 7] = fmaxf(mx[k & 7], s[k]);
-      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      for (int e = 0; e < 8; ++e) mx[e] = fmax3(mx[e], s[24 + e], s[32 + e]);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = fmax3(mx[e], s[40 + e], s[48 + e]);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[56 + e]);
+      const float mh = fmaxf(fmax3(mx[0], mx[1], mx[2]),
+                             fmax3(fmax3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
+      ctl.red_max[j & 1][half][t] = mh;
+      pair_bar_sync(quarter);
+      const float mt = fmaxf(mh, ctl.red_max[j & 1][half ^ 1][t]);
       // Raise the reference maximum on the first finite value, or when the tile maximum
       // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
+      // Both warps of a row take the same decision from the same values.
       float m_new = m_run;
       if (m_run == -INFINITY) m_new = mt;
       else if ((mt - m_run) * sl > kRescaleLog2) m_new = mt;
       const bool rescale = (m_new != m_run) && (m_run != -INFINITY);
       const float alpha = rescale ? ex2_approx((m_run - m_new) * sl) : 1.f;
-      if (__any_sync(0xffffffffu, rescale)) {
-        // PV_{j-1} may still be accumulating into O: wait for it first
-        ok = mbar_wait(&ctl.pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1);
+      const float mL = (m_new == -INFINITY) ? 0.f : m_new * sl;
+      uint32_t pk[32];
+      const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
+      uint64_t acc[4] = {0, 0, 0, 0};  // four packed partial sums (bit pattern 0 = +0.0f)
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        float x0, x1;
+        f2_unpack(f2_fma(f2_pack(s[2 * e], s[2 * e + 1]), sl2, nmL2), x0, x1);
+        const float a = ex2_approx(x0);
+        const float c = ex2_approx(x1);
+        const uint64_t pc = f2_pack(a, c);
+        acc[e & 3] = f2_add(acc[e & 3], pc);
+        pk[e] = pack_bf16x2(a, c);
+      }
+      float ls[4];
+      {
+        float a0, a1, b0, b1;
+        f2_unpack(f2_add(acc[0], acc[1]), a0, a1);
+        f2_unpack(f2_add(acc[2], acc[3]), b0, b1);
+        ls[0] = a0; ls[1] = a1; ls[2] = b0; ls[3] = b1;
+      }
+      // P_j replaces P_{j-1}, and O may be rescaled, once PV_{j-1} has completed
+      if (j > 0) {
+        ok = mbar_wait(&ctl.pv_done, (j - 1) & 1);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
+      }
+      if (__any_sync(0xffffffffu, rescale)) {
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
+        for (int c = 0; c < D / 64; ++c) {  // this warp's half of the O columns
           uint32_t r[32];
-          tmem_ld32(tO + lane_off + c * 32, r);
+          const uint32_t col = tO + lane_off + half * (D / 2) + 32 * c;
+          tmem_ld32(col, r);
           tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-          tmem_st32(tO + lane_off + c * 32, r);
+          tmem_st32(col, r);
         }
       }
-      l_run *= alpha;
+      l_run = l_run * alpha + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
       m_run = m_new;
-      const float mL = (m_run == -INFINITY) ? 0.f : m_run * sl;
-      uint32_t pk[32];
-      float ls[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        const float a = ex2_approx(fmaf(s[2 * e], sl, -mL));
-        const float c = ex2_approx(fmaf(s[2 * e + 1], sl, -mL));
-        ls[e & 3] += a + c;
-        pk[e] = pack_bf16x2(a, c);
-      }
-      l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      tmem_st32(ctl.tmem_base + b * kTN + lane_off, pk);
+      tmem_st32(tP + lane_off + 32 * half, pk);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.p_full[b]);
+      if (lane == 0) mbar_arrive(&ctl.p_full);
     }
     if (ok) ok = mbar_wait(&ctl.o_full, 0);
     const bool wok = __all_sync(0xffffffffu, ok);
     if (!wok && lane == 0) flag_timeout(p, ctl);
-    // O row / row sum -> bf16 into shared memory (the Q tile is no longer read once o_full
-    // has completed), 16-byte chunks XOR-swizzled by row; then the 128 threads store whole
-    // rows, coalesced. Every softmax warp reaches the named barrier on every path.
+    // O row / row sum -> bf16 into shared memory (the K stages are no longer read once
+    // o_full has completed), 16-byte chunks XOR-swizzled by row; then the 256 softmax
+    // threads store whole rows, coalesced. Every softmax warp reaches the named barriers
+    // on every path.
+    ctl.red_sum[half][t] = l_run;
+    softmax_bar_sync();
     constexpr int kChunks = D / 8;  // 16-byte chunks per output row
     const int r = q0 + t;
-    uint4* stage = reinterpret_cast<uint4*>(sQ);
+    uint4* stage = reinterpret_cast<uint4*>(sK);  // 128 rows x D bf16 <= one K stage
     if (wok) {
       tc_fence_after();
-      const float inv_l = 1.0f / l_run;
+      const float inv_l = 1.0f / (ctl.red_sum[0][t] + ctl.red_sum[1][t]);
 #pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
+      for (int c = 0; c < D / 64; ++c) {
         uint32_t rr[32];
-        tmem_ld32(tO + lane_off + c * 32, rr);
+        tmem_ld32(tO + lane_off + half * (D / 2) + 32 * c, rr);
         tmem_wait_ld();
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
@@ -588,17 +686,18 @@ __global__ void __launch_bounds__(kTcThreads, 2)
           u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
           u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
           u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
-          const int chunk = c * 4 + v;
+          const int chunk = half * (kChunks / 2) + c * 4 + v;
           stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
         }
       }
     }
-    ctl.store_row[t] = (wok && q.store && r < rows_seq) ? 1 : 0;
-    sm_bar_sync();
+    if (half == 0) ctl.store_row[t] = (wok && q.store && r < rows_seq) ? 1 : 0;
+    softmax_bar_sync();
     if (!*abort_flag) {
       __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o);
+      const int tid = threadIdx.x;  // 0 .. 255
 #pragma unroll 4
-      for (int idx = t; idx < kBM * kChunks; idx += 128) {
+      for (int idx = tid; idx < kBM * kChunks; idx += 32 * kSoftmaxWarps) {
         const int row = idx / kChunks, chunk = idx % kChunks;
         if (ctl.store_row[row]) {
           const uint4 u = stage[row * kChunks + (chunk ^ (row & (kChunks - 1)))];
@@ -611,7 +710,7 @@ __global__ void __launch_bounds__(kTcThreads, 2)
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kWPV) {
     tc_fence_after();
     tmem_dealloc<kTmemCols>(ctl.tmem_base);
   }
@@ -716,15 +815,14 @@ cudaError_t ensure_smem_attr(F* kernel, size_t bytes, std::atomic<uint64_t>& don
 template <int D>
 cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
   static std::atomic<uint64_t> attr_done{0};
-  CUtensorMap mq, mk, mv;
-  if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM) ||
-      !make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
+  CUtensorMap mk, mv;
+  if (!make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
       !make_map(&mv, p.v, p.hkv, D, p.total_rows, kTN))
     return cudaErrorInvalidValue;
   const size_t smem = tc_smem_bytes<D>();
   cudaError_t e = ensure_smem_attr(attn_tc<D>, smem, attr_done);
   if (e != cudaSuccess) return e;
-  attn_tc<D><<<p.total_work, kTcThreads, smem, stream>>>(p, mq, mk, mv);
+  attn_tc<D><<<p.total_work, kTcThreads, smem, stream>>>(p, mk, mv);
   return cudaGetLastError();
 }
 
