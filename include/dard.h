@@ -16,7 +16,8 @@
  *   - Pointers named "device" are CUDA device memory owned by the caller; pointers named
  *     "host" are ordinary host memory owned by the caller and read during the call only.
  *   - Every call is asynchronous on the given stream; nothing is synchronised.
- *   - The library never allocates memory. Scratch space is passed in by the caller.
+ *   - The library never allocates memory. Scratch space is passed in by the caller, or
+ *     (dard_score_and_transition_noalloc) is a fixed array inside the library.
  *   - Argument and shape errors are detected on the host and returned before any launch;
  *     nothing is launched when a call returns an error. A failed launch returns
  *     DARD_ERR_CUDA (the CUDA error string is available from dard_last_error()).
@@ -164,6 +165,35 @@ size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs);
 /* Logits pointers must be 16-byte aligned and row_stride * element size a multiple of 16.
  * Errors: DARD_ERR_NULL, _SHAPE, _VALUE, _ALIGN, _WORKSPACE, _CUDA. */
 dard_status dard_score_and_transition(const dard_score_args* args, void* stream);
+
+/* ------------------------------------------------------------------------------------- *
+ * dard_score_and_transition_noalloc: the same scoring and transition, with the scratch
+ * inside the library. The paper has no counterpart: this is an interface addition.
+ *
+ * Who needs it: a caller that only holds the buffers another component handed to it (a
+ * plug-in inside an inference server, a C host program driving a model it did not load)
+ * and has no device allocator, or one whose device memory is planned in advance so that no
+ * call may ask for more. Such a caller cannot provide `workspace`; this entry point needs
+ * none and neither allocates nor frees device memory.
+ *
+ * Arguments, outputs and errors are those of dard_score_and_transition, except that
+ * `workspace` and `workspace_bytes` are ignored. The scratch is a fixed array of
+ * DARD_SCORE_NOALLOC_MAX_ROWS bytes in the library's device memory (one byte per block row,
+ * the outcome of the verification pass). A call with more block rows (sum of block_len)
+ * than that returns DARD_ERR_WORKSPACE before any launch; use dard_score_and_transition
+ * with a workspace for it. Nothing in the array needs to start at zero: every call writes
+ * each byte it reads before reading it.
+ *
+ * The first call on each device (the device current at the call) looks up the array's
+ * address there once (cudaGetSymbolAddress) and caches it; make that first call before any
+ * stream capture on that device. A failed lookup returns DARD_ERR_CUDA.
+ *
+ * There is one array per device, shared by every call on it: calls whose kernels can
+ * overlap on one device (different streams, different host threads) race on it and may
+ * return wrong results. Order them (one stream, or events between streams).
+ * ------------------------------------------------------------------------------------- */
+#define DARD_SCORE_NOALLOC_MAX_ROWS 8192
+dard_status dard_score_and_transition_noalloc(const dard_score_args* args, void* stream);
 
 /* Human-readable name of a status code; never NULL. */
 const char* dard_status_string(dard_status s);

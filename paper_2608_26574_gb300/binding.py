@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_PKG, "libdard.so")
 DARD_F32, DARD_BF16 = 0, 1
 STATUS_BAD_STATE, STATUS_BAD_SHADOW, STATUS_INVALID_ROW, STATUS_TIMEOUT = 0x1, 0x2, 0x4, 0x8
 MAX_SEQS, MAX_BLOCK = 256, 128
+SCORE_NOALLOC_MAX_ROWS = 8192
 
 _I32P = ctypes.POINTER(ctypes.c_int32)
 
@@ -58,6 +59,8 @@ _lib = None
 EXPORTS = {
     "dard_step_attention": (ctypes.c_int, [ctypes.POINTER(AttnArgs), ctypes.c_void_p]),
     "dard_score_and_transition": (ctypes.c_int, [ctypes.POINTER(ScoreArgs), ctypes.c_void_p]),
+    "dard_score_and_transition_noalloc": (ctypes.c_int, [ctypes.POINTER(ScoreArgs),
+                                                         ctypes.c_void_p]),
     "dard_score_workspace_size": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
     "dard_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "dard_last_error": (ctypes.c_char_p, []),
@@ -175,3 +178,26 @@ def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, ta
     a.workspace_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     _check(lib().dard_score_and_transition(ctypes.byref(a), _stream(stream)),
            "dard_score_and_transition")
+
+
+def dard_score_and_transition_noalloc(logits_x, logits_s, block_len, state_in, tau_c, tau_u,
+                                      lam, p0, conf, token, state_out, w_out=None, counts=None,
+                                      status=None, stream=None):
+    """``dard_score_and_transition`` without a workspace: the library's built-in scratch
+    (at most ``SCORE_NOALLOC_MAX_ROWS`` block rows; calls that overlap on one device race)."""
+    block_len = _host_i32(block_len)
+    if logits_x.stride(0) != logits_s.stride(0) or logits_x.shape != logits_s.shape:
+        raise ValueError("logits_x and logits_s need the same shape and row pitch")
+    a = ScoreArgs()
+    a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
+    a.dtype = _dtype_code(logits_s)
+    a.vocab = logits_s.shape[1]
+    a.row_stride = logits_s.stride(0)
+    a.num_seqs = len(block_len)
+    a.block_len = block_len.ctypes.data_as(_I32P)
+    a.state_in = _ptr(state_in)
+    a.tau_c, a.tau_u, a.lambda_, a.p0 = tau_c, tau_u, lam, p0
+    a.conf, a.token, a.state_out = _ptr(conf), _ptr(token), _ptr(state_out)
+    a.w_out, a.counts, a.status = _ptr(w_out), _ptr(counts), _ptr(status)
+    _check(lib().dard_score_and_transition_noalloc(ctypes.byref(a), _stream(stream)),
+           "dard_score_and_transition_noalloc")

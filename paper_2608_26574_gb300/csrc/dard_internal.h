@@ -73,5 +73,7 @@ constexpr int kScoreMaxSplit = 16;  // CTAs per row = thread-block cluster size
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs);
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
                          char* err, size_t err_len);
+// Records the message returned by dard_last_error() on this thread and returns `s`.
+dard_status report(dard_status s, const char* fmt, ...);
 
 }  // namespace dard

@@ -1,0 +1,72 @@
+// dard_noalloc.cu - dard_score_and_transition_noalloc: the scoring call with its scratch in a
+// fixed array inside the library, for callers that cannot hand device memory to it.
+//
+// The only scratch the scoring kernels use is one byte per block row (the promotion /
+// demotion outcome of pass 1, read by pass 2). Here that byte array is a file-scope
+// __device__ array of DARD_SCORE_NOALLOC_MAX_ROWS bytes. Its address on a device is looked up
+// once (cudaGetSymbolAddress, with that device current) on the first call made on that
+// device, cached per device, and then passed as the workspace of dard_score_and_transition,
+// whose kernels and validation run unchanged. No call allocates or frees device memory.
+#include <mutex>
+
+#include "dard_internal.h"
+
+namespace {
+
+__device__ __align__(256) uint8_t g_score_scratch[DARD_SCORE_NOALLOC_MAX_ROWS];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of g_score_scratch on the current device (looked up on first use).
+cudaError_t scratch_on_current_device(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_score_scratch);
+    if (e != cudaSuccess) return e;
+    if (ptr == nullptr) return cudaErrorInvalidSymbol;
+    g_scratch_ptr[dev] = ptr;
+  }
+  *out = g_scratch_ptr[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" dard_status dard_score_and_transition_noalloc(const dard_score_args* a, void* stream) {
+  using namespace dard;
+  if (!a) return report(DARD_ERR_NULL, "args is NULL");
+  // Sizes that dard_score_and_transition itself rejects are passed on to it for its message.
+  long long rows = 0;
+  bool sizes_ok = a->block_len != nullptr && a->num_seqs >= 1 && a->num_seqs <= DARD_MAX_SEQS;
+  for (int s = 0; sizes_ok && s < a->num_seqs; ++s) {
+    const int B = a->block_len[s];
+    sizes_ok = B >= 0 && B <= DARD_MAX_BLOCK;
+    rows += B;
+  }
+  dard_score_args b = *a;
+  b.workspace = nullptr;
+  b.workspace_bytes = 0;
+  if (sizes_ok && rows > 0) {
+    if (rows > DARD_SCORE_NOALLOC_MAX_ROWS)
+      return report(DARD_ERR_WORKSPACE,
+                    "%lld block rows exceed the %d rows the built-in scratch of "
+                    "dard_score_and_transition_noalloc holds; use dard_score_and_transition "
+                    "with a workspace",
+                    rows, DARD_SCORE_NOALLOC_MAX_ROWS);
+    void* scratch = nullptr;
+    const cudaError_t e = scratch_on_current_device(&scratch);
+    if (e != cudaSuccess)
+      return report(DARD_ERR_CUDA, "looking up the built-in scratch failed: %s",
+                    cudaGetErrorString(e));
+    b.workspace = scratch;
+    b.workspace_bytes = sizeof(g_score_scratch);
+  }
+  return dard_score_and_transition(&b, stream);
+}
