@@ -111,15 +111,19 @@ dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
   std::vector<int> order(a->num_seqs);
   std::iota(order.begin(), order.end(), 0);
   std::stable_sort(order.begin(), order.end(), [&](int x, int y) { return cost[x] > cost[y]; });
-  long long work = 0;
+  long long work = 0, pairs = 0;
   for (int r = 0; r < a->num_seqs; ++r) {
     p.order[r] = order[r];
     p.work_prefix[r] = static_cast<int32_t>(work);
+    p.pair_prefix[r] = static_cast<int32_t>(pairs);
     work += static_cast<long long>(p.seq[order[r]].n_qtiles) * a->hq;
+    pairs += static_cast<long long>((p.seq[order[r]].n_qtiles + 1) / 2) * a->hq;
     if (work > (1ll << 31) - 1) return fail(DARD_ERR_SHAPE, "too many work items");
   }
   p.work_prefix[a->num_seqs] = static_cast<int32_t>(work);
+  p.pair_prefix[a->num_seqs] = static_cast<int32_t>(pairs);
   p.total_work = static_cast<int32_t>(work);
+  p.total_pairs = static_cast<int32_t>(pairs);
   p.total_rows = static_cast<int32_t>(rows);
   p.state = a->state;
   p.prev_conf = a->prev_conf;

@@ -8,17 +8,20 @@
 // so the mask is evaluated only on the (at most three) tiles that contain block keys,
 // shadow keys or the ragged end of the sequence.
 //
-// bf16 path (attn_tc): one CTA per SM = 128 query rows of one (sequence, head); 6 warps:
-//   warps 0-3  softmax and epilogue, thread t owns query row t (= TMEM lane t);
-//   warp 4     TMA producer: Q once, then K and V tiles of 64 keys through 4 stages each,
-//              with L2 prefetches a few tiles further ahead;
-//   warp 5     TMEM allocator and PV issuer: O += P_j V_j with P_j (bf16) read from TMEM
-//              where the softmax warps wrote it over S_j;
-//   warp 6     S issuer: S_j = Q K_j^T (tcgen05, Q from TMEM, K from shared memory) into a
-//              ring of four 64-column TMEM buffers. With its own issuing thread S runs up
-//              to four tiles ahead of the softmax and is never held up behind a PV wait.
+// bf16 path (attn_tc): one CTA per SM = 128 query rows of one (sequence, head); 11 warps:
+//   warps 0-7  softmax and epilogue: warps w and w + 4 share TMEM lane quarter w (query
+//              rows 32w .. 32w + 31), each taking 64 of a tile's 128 key columns;
+//   warp 8     TMA producer: K and V tiles of 128 keys through 3 stages each, with L2
+//              prefetches a few tiles further ahead;
+//   warp 9     TMEM allocator and PV issuer: O += P_j V_j with P_j (bf16) read from TMEM,
+//              where the softmax warps wrote it over the first half of each warp's S_j
+//              columns;
+//   warp 10    S issuer: S_j = Q K_j^T (tcgen05, Q from TMEM, K from shared memory) into a
+//              ring of two 128-column TMEM buffers, each reused once the PV that reads the
+//              P stored in it has completed.
 // The softmax threads write their query rows into TMEM (bf16 pairs, the A-operand layout)
-// at the start, so shared-memory bandwidth goes to K and V only.
+// at the start, so shared-memory bandwidth goes to K and V only. With P in its own S
+// buffer, the softmax of tile j + 1 never waits for the PV of tile j.
 // The online softmax keeps a per-row running maximum and rescales O in TMEM only when the
 // maximum grows by more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
 // fp32 path (attn_simt): CUDA-core kernel, one warp per query row, same mask logic.
@@ -31,6 +34,7 @@
 #include <atomic>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <mutex>
 #include <numeric>
 #include <vector>
@@ -42,9 +46,9 @@ namespace dard {
 namespace {
 
 constexpr int kBM = 128;  // query rows per CTA
-constexpr int kTcThreads = 352;  // 8 softmax warps, producer, PV issuer, S issuer
-constexpr uint32_t kTmemCols = 512;  // S/P ring: 2 x 128 columns [0, 256); O: [256, 256 + D);
-                                     // Q (bf16 pairs): [384, 384 + D / 2)
+constexpr int kTc1Threads = 352;  // attn_tc1: 8 softmax warps, producer, PV issuer, S issuer
+constexpr int kTc2Threads = 320;  // attn_tc2: 2 x 4 softmax warps, TMA producer, MMA issuer
+constexpr uint32_t kTmemCols = 512;  // every TMEM column of the SM
 constexpr float kRescaleLog2 = 8.0f;
 
 // Per-CTA copy of the current block: states, confidences, the shadow maps, and the same
@@ -82,6 +86,21 @@ __device__ __forceinline__ void decode_work(const AttnParams& p, int w, int& seq
   const int local = w - p.work_prefix[lo];
   h = local % p.hq;
   qt = local / p.hq;
+}
+
+// The same over pairs of query tiles (the tensor-core path): work item w is query-tile pair
+// pr of head h of sequence seq.
+__device__ __forceinline__ void decode_pair(const AttnParams& p, int w, int& seq, int& pr,
+                                            int& h) {
+  int lo = 0, hi = p.num_seqs;  // pair_prefix[lo] <= w < pair_prefix[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (p.pair_prefix[mid] <= w) lo = mid; else hi = mid;
+  }
+  seq = p.order[lo];
+  const int local = w - p.pair_prefix[lo];
+  h = local % p.hq;
+  pr = local / p.hq;
 }
 
 // The block's per-position data as one thread fetches it from global memory (thread t:
@@ -316,15 +335,28 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+constexpr int kQT = 2;   // query tiles per CTA (the same sequence and head)
+constexpr int kNK = 2;   // TMA stages for K
+constexpr int kNV = 2;   // TMA stages for V
+constexpr int kWProd = 2 * kQT * 2;  // warp 8: TMA producer
+constexpr int kWMma = kWProd + 1;    // warp 9: TMEM allocator and MMA issuer
+
+// Named barriers: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = the 8 softmax warps,
+// then per kernel: attn_tc1 3 + q = the two warps sharing TMEM lane quarter q; attn_tc2
+// 3 + q = the four warps of query tile q.
+__device__ __forceinline__ void softmax_bar_sync() {
+  asm volatile("bar.sync 2, 256;" ::: "memory");
+}
+__device__ __forceinline__ void tile_bar_sync(int q) {
+  asm volatile("bar.sync %0, 128;" ::"r"(3 + q) : "memory");
+}
+
 constexpr int kNS = 2;   // S buffers in TMEM (a ring of 128-column buffers)
 constexpr int kNKV = 3;  // TMA stages for K and for V
 constexpr int kSoftmaxWarps = 8;  // two warps per query row, 64 key columns each
 
-// Named barriers: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = all softmax warps,
-// 3 + q = the two warps (q and q + 4) that share TMEM lane quarter q.
-__device__ __forceinline__ void softmax_bar_sync() {
-  asm volatile("bar.sync 2, 256;" ::: "memory");
-}
+// Named barriers of attn_tc1: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = all
+// softmax warps, 3 + q = the two warps (q and q + 4) that share TMEM lane quarter q.
 __device__ __forceinline__ void pair_bar_sync(int quarter) {
   asm volatile("bar.sync %0, 64;" ::"r"(3 + quarter) : "memory");
 }
@@ -333,7 +365,7 @@ __device__ __forceinline__ void pair_bar_sync(int quarter) {
 // and waits for parity (j / ring) & 1. A waiter is never more than one phase behind the
 // phase it waits for (the parity would alias otherwise): each wait for use u of a slot is
 // preceded, in the same thread or through a chain of waits, by the completion of use u - 1.
-struct __align__(16) TcCtl {
+struct __align__(16) Tc1Ctl {
   uint64_t q_full, o_full, p_full, pv_done;
   uint64_t k_full[kNKV], k_empty[kNKV], v_full[kNKV], v_empty[kNKV];
   uint64_t s_full[kNS], s_free[kNS];
@@ -347,19 +379,19 @@ struct __align__(16) TcCtl {
 };
 
 template <int D>
-constexpr size_t tc_smem_bytes() {
+constexpr size_t tc1_smem_bytes() {
   // alignment slack + kNKV stages each of K and V (128 rows) + control
-  return 1024 + 2 * kNKV * static_cast<size_t>(kTN) * D * 2 + sizeof(TcCtl);
+  return 1024 + 2 * kNKV * static_cast<size_t>(kTN) * D * 2 + sizeof(Tc1Ctl);
 }
 
-__device__ __forceinline__ void flag_timeout(const AttnParams& p, TcCtl& ctl) {
+__device__ __forceinline__ void flag_timeout(const AttnParams& p, Tc1Ctl& ctl) {
   ctl.abort = 1;
   if (p.status) atomicOr(p.status, DARD_STATUS_TIMEOUT);
 }
 
 template <int D>
-__global__ void __launch_bounds__(kTcThreads, 1)
-    attn_tc(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmk,
+__global__ void __launch_bounds__(kTc1Threads, 1)
+    attn_tc1(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmk,
             const __grid_constant__ CUtensorMap tmv) {
   constexpr int kSub = D / 64;                 // 128-byte (64 x bf16) column blocks
   constexpr uint32_t kKSub = kTN * 128;        // one 128-row x 128-byte swizzled block
@@ -370,7 +402,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sK = base;                  // kNKV stages
   uint8_t* sV = sK + kNKV * kKVBytes;  // kNKV stages
-  TcCtl& ctl = *reinterpret_cast<TcCtl*>(sV + kNKV * kKVBytes);
+  Tc1Ctl& ctl = *reinterpret_cast<Tc1Ctl*>(sV + kNKV * kKVBytes);
 
   int seq, qt, h;
   decode_work(p, blockIdx.x, seq, qt, h);
@@ -716,6 +748,388 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
+
+// One query row's pass over a 128-key S tile in TMEM (columns tS .. tS + 127 of its lane),
+// 64 columns at a time; kMasked applies the visibility bits (vis0: keys 0-63, vis1: 64-127).
+template <bool kMasked>
+__device__ __forceinline__ float tile_row_max(uint32_t tS, uint64_t vis0, uint64_t vis1) {
+  float mx[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
+#pragma unroll
+  for (int hh = 0; hh < 2; ++hh) {
+    uint32_t r0[32], r1[32];
+    tmem_ld32(tS + 64 * hh, r0);
+    tmem_ld32(tS + 64 * hh + 32, r1);
+    tmem_wait_ld();
+    const uint64_t vis = hh ? vis1 : vis0;
+#pragma unroll
+    for (int e = 0; e < 32; e += 2) {
+      float x0 = __uint_as_float(r0[e]), x1 = __uint_as_float(r0[e + 1]);
+      float y0 = __uint_as_float(r1[e]), y1 = __uint_as_float(r1[e + 1]);
+      if (kMasked) {
+        x0 = ((vis >> e) & 1ull) ? x0 : -INFINITY;
+        x1 = ((vis >> (e + 1)) & 1ull) ? x1 : -INFINITY;
+        y0 = ((vis >> (32 + e)) & 1ull) ? y0 : -INFINITY;
+        y1 = ((vis >> (33 + e)) & 1ull) ? y1 : -INFINITY;
+      }
+      mx[(e >> 1) & 7] = fmaxf(fmax3(mx[(e >> 1) & 7], x0, x1), fmaxf(y0, y1));
+    }
+  }
+  return fmaxf(fmax3(mx[0], mx[1], mx[2]), fmax3(fmax3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
+}
+
+// P = 2^(s * sl - mL) for the row's 128 keys as bf16 pairs: keys 64 hh .. 64 hh + 63 go to
+// columns tS + 32 hh .. tS + 32 hh + 31, over S values this thread has already read. The
+// fp32 values are summed into acc (four packed partial sums).
+template <bool kMasked>
+__device__ __forceinline__ void tile_row_exp(uint32_t tS, uint64_t vis0, uint64_t vis1,
+                                             uint64_t sl2, uint64_t nmL2, uint64_t (&acc)[4]) {
+#pragma unroll
+  for (int hh = 0; hh < 2; ++hh) {
+    uint32_t r0[32], r1[32];
+    tmem_ld32(tS + 64 * hh, r0);
+    tmem_ld32(tS + 64 * hh + 32, r1);
+    tmem_wait_ld();
+    const uint64_t vis = hh ? vis1 : vis0;
+    uint32_t pk[32];
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      float s0 = __uint_as_float(e < 16 ? r0[2 * e] : r1[2 * e - 32]);
+      float s1 = __uint_as_float(e < 16 ? r0[2 * e + 1] : r1[2 * e - 31]);
+      if (kMasked) {
+        s0 = ((vis >> (2 * e)) & 1ull) ? s0 : -INFINITY;
+        s1 = ((vis >> (2 * e + 1)) & 1ull) ? s1 : -INFINITY;
+      }
+      float x0, x1;
+      f2_unpack(f2_fma(f2_pack(s0, s1), sl2, nmL2), x0, x1);
+      const float a = ex2_approx(x0);
+      const float c = ex2_approx(x1);
+      acc[e & 3] = f2_add(acc[e & 3], f2_pack(a, c));
+      pk[e] = pack_bf16x2(a, c);
+    }
+    tmem_st32(tS + 32 * hh, pk);
+  }
+}
+
+// Barrier protocol. Every barrier completes one phase per use; use u waits for parity
+// (u / ring) & 1, and no waiter is ever two phases behind (the parity would alias):
+// each wait for use u is preceded, in the same thread or through a chain of waits, by the
+// completion of use u - ring.
+struct __align__(16) Tc2Ctl {
+  uint64_t q_full;  // both query tiles landed
+  uint64_t k_full[kNK], k_empty[kNK], v_full[kNV], v_empty[kNV];
+  uint64_t s_full[kQT];   // S_q(j) landed in TMEM
+  uint64_t p_full[kQT];   // the softmax of tile q stored P_q(j) over S_q(j)
+  uint64_t pv_done[kQT];  // PV_q(j) completed: S_q's columns may take S_q(j + 1)
+  uint64_t o_full[kQT];   // the last PV_q completed
+  uint32_t tmem_base;
+  int32_t abort;
+  BlockInfo bi;
+  uint8_t store_row[kQT][kBM];  // epilogue: rows of each tile that are written
+};
+
+template <int D>
+constexpr size_t tc2_smem_bytes() {
+  // alignment slack + kQT query tiles + kNK K stages + kNV V stages (128 rows each) + control
+  return 1024 + (kQT + kNK + kNV) * static_cast<size_t>(kTN) * D * 2 + sizeof(Tc2Ctl);
+}
+
+__device__ __forceinline__ void flag_timeout(const AttnParams& p, Tc2Ctl& ctl) {
+  ctl.abort = 1;
+  if (p.status) atomicOr(p.status, DARD_STATUS_TIMEOUT);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kTc2Threads, 1)
+    attn_tc2(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmq,
+            const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv) {
+  constexpr int kSub = D / 64;                   // 128-byte (64 x bf16) column blocks
+  constexpr uint32_t kKSub = kTN * 128;          // one 128-row x 128-byte swizzled block
+  constexpr uint32_t kTileBytes = kSub * kKSub;  // one 128-row tile of Q, K or V
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sQ = base;                     // kQT query tiles
+  uint8_t* sK = sQ + kQT * kTileBytes;    // kNK stages
+  uint8_t* sV = sK + kNK * kTileBytes;    // kNV stages
+  Tc2Ctl& ctl = *reinterpret_cast<Tc2Ctl*>(sV + kNV * kTileBytes);
+
+  int seq, pr, h;
+  decode_pair(p, blockIdx.x, seq, pr, h);
+  const SeqDesc sd = p.seq[seq];
+  const int rows_seq = sd.n_orig + sd.slen;
+  const int n_kt = (rows_seq + kTN - 1) / kTN;
+  const int qt0 = kQT * pr;                       // first query tile of this CTA
+  const int nq = min(kQT, sd.n_qtiles - qt0);     // 1 or 2 query tiles
+  const int g = h / (p.hq / p.hkv);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row0 = sd.row_base;
+
+  auto load_kv = [&](int j, bool k_or_v) {
+    const int b = j % (k_or_v ? kNK : kNV);
+    uint64_t* bar = k_or_v ? &ctl.k_full[b] : &ctl.v_full[b];
+    uint8_t* dst = (k_or_v ? sK : sV) + b * kTileBytes;
+    const void* map = k_or_v ? static_cast<const void*>(&tmk) : static_cast<const void*>(&tmv);
+    mbar_arrive_expect_tx(bar, kTileBytes);
+#pragma unroll
+    for (int s = 0; s < kSub; ++s)
+      tma_load_2d(dst + s * kKSub, map, bar, g * D + s * 64, row0 + j * kTN);
+  };
+  auto prefetch_kv = [&](int j) {
+#pragma unroll
+    for (int s = 0; s < kSub; ++s) {
+      tma_prefetch_l2_2d(&tmk, g * D + s * 64, row0 + j * kTN);
+      tma_prefetch_l2_2d(&tmv, g * D + s * 64, row0 + j * kTN);
+    }
+  };
+  // The producer lane initialises the barriers and issues the query tiles and the first
+  // K/V stages at once; the other threads touch the barriers only after the block sync.
+  if (warp == kWProd && lane == 0) {
+    mbar_init(&ctl.q_full, 1);
+    for (int b = 0; b < kNK; ++b) {
+      mbar_init(&ctl.k_full[b], 1);
+      mbar_init(&ctl.k_empty[b], 1);
+    }
+    for (int b = 0; b < kNV; ++b) {
+      mbar_init(&ctl.v_full[b], 1);
+      mbar_init(&ctl.v_empty[b], 1);
+    }
+    for (int q = 0; q < kQT; ++q) {
+      mbar_init(&ctl.s_full[q], 1);
+      mbar_init(&ctl.p_full[q], 4);
+      mbar_init(&ctl.pv_done[q], 1);
+      mbar_init(&ctl.o_full[q], 1);
+    }
+    ctl.abort = 0;
+    fence_barrier_init();
+    tma_prefetch_desc(&tmq);
+    tma_prefetch_desc(&tmk);
+    tma_prefetch_desc(&tmv);
+    mbar_arrive_expect_tx(&ctl.q_full, nq * kTileBytes);
+    for (int q = 0; q < nq; ++q) {
+#pragma unroll
+      for (int s = 0; s < kSub; ++s)
+        tma_load_2d(sQ + q * kTileBytes + s * kKSub, &tmq, &ctl.q_full, h * D + s * 64,
+                    row0 + (qt0 + q) * kBM);
+    }
+    for (int j = 0; j < kNK && j < n_kt; ++j) load_kv(j, true);
+    for (int j = 0; j < kNV && j < n_kt; ++j) load_kv(j, false);
+    for (int j = kNK; j < kNK + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
+  }
+  if (warp == kWMma) {
+    tmem_alloc<kTmemCols>(&ctl.tmem_base);
+    tmem_relinquish();
+  }
+  BlockFetch bf{-1, 0.f, -1};
+  if (warp < 4) bf = fetch_block_info(p, sd);  // in flight across the block sync
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  // TMEM columns: S_q / P_q [128 q, 128 q + 128) (P_q(j) as bf16 pairs over the first 64),
+  // O_q [256 + D q, 256 + D q + D)
+  const uint32_t tS0 = ctl.tmem_base;
+  const uint32_t tO0 = ctl.tmem_base + kQT * kTN;
+  volatile int32_t* abort_flag = &ctl.abort;
+
+  if (warp == kWProd) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int last_k = min(n_kt, kNK) - 1, last_v = min(n_kt, kNV) - 1;
+      for (int j = min(kNK, kNV); j < n_kt && !*abort_flag; ++j) {
+        if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
+        if (j >= kNK) {
+          const int b = j % kNK;
+          if (!mbar_wait(&ctl.k_empty[b], ((j - kNK) / kNK) & 1)) { flag_timeout(p, ctl); break; }
+          load_kv(j, true);
+          last_k = j;
+        }
+        if (j >= kNV) {
+          const int b = j % kNV;
+          if (!mbar_wait(&ctl.v_empty[b], ((j - kNV) / kNV) & 1)) { flag_timeout(p, ctl); break; }
+          load_kv(j, false);
+          last_v = j;
+        }
+      }
+      if (*abort_flag) {
+        // let the copies already in flight land before shared memory is released
+        if (last_k >= 0) mbar_wait(&ctl.k_full[last_k % kNK], (last_k / kNK) & 1);
+        if (last_v >= 0) mbar_wait(&ctl.v_full[last_v % kNV], (last_v / kNV) & 1);
+        mbar_wait(&ctl.q_full, 0);
+      }
+    }
+  } else if (warp == kWMma) {
+    // ------------------------------------------------------------ MMA issuer
+    // Tensor-pipe order: S_0(0) S_1(0) | PV_0(j) S_0(j+1) PV_1(j) S_1(j+1) | ... The softmax
+    // of tile 0 runs while the pipe does PV_1 and S_1, and the other way round. S_q(j+1)
+    // overwrites the P_q(j) that PV_q(j) reads, so it is issued once PV_q(j) has completed.
+    if (lane == 0) {
+      constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
+      constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
+      const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK), av = smem_u32(sV);
+      auto issue_s = [&](int q, int j) {
+        const uint32_t qaddr = aq + q * kTileBytes, kaddr = ak + (j % kNK) * kTileBytes;
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (ks >> 2) * kKSub + (ks & 3) * 32;
+          mma_ss(tS0 + q * kTN, smem_desc_sw128(qaddr + off, 16, 1024),
+                 smem_desc_sw128(kaddr + off, 16, 1024), kIdS, ks > 0);
+        }
+        mma_commit(&ctl.s_full[q]);
+      };
+      auto issue_pv = [&](int q, int j) {
+        const uint32_t vaddr = av + (j % kNV) * kTileBytes;
+#pragma unroll
+        for (int ks = 0; ks < kTN / 16; ++ks)
+          mma_ts(tO0 + q * D, tS0 + q * kTN + ks * 8,
+                 smem_desc_sw128(vaddr + ks * 2048, kKSub, 1024), kIdO,
+                 (j > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&ctl.pv_done[q]);
+        if (j == n_kt - 1) mma_commit(&ctl.o_full[q]);
+      };
+      bool ok = mbar_wait(&ctl.q_full, 0) && mbar_wait(&ctl.k_full[0], 0);
+      if (ok) {
+        tc_fence_after();
+        for (int q = 0; q < nq; ++q) issue_s(q, 0);
+        mma_commit(&ctl.k_empty[0]);
+      }
+      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
+        const bool more = j + 1 < n_kt;
+        ok = mbar_wait(&ctl.v_full[j % kNV], (j / kNV) & 1);
+        if (ok && more) ok = mbar_wait(&ctl.k_full[(j + 1) % kNK], ((j + 1) / kNK) & 1);
+        for (int q = 0; q < nq && ok; ++q) {
+          ok = mbar_wait(&ctl.p_full[q], j & 1);
+          if (!ok) break;
+          tc_fence_after();
+          issue_pv(q, j);
+          if (q == nq - 1) mma_commit(&ctl.v_empty[j % kNV]);
+          if (more) {
+            ok = mbar_wait(&ctl.pv_done[q], j & 1);
+            if (!ok) break;
+            tc_fence_after();
+            issue_s(q, j + 1);
+            if (q == nq - 1) mma_commit(&ctl.k_empty[(j + 1) % kNK]);
+          }
+        }
+      }
+      if (!ok) flag_timeout(p, ctl);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax + epilogue
+    // Warps 4q .. 4q + 3 own query tile q; thread t = query row t of the tile (TMEM lane t).
+    const int q = warp >> 2, quarter = warp & 3;
+    const int t = quarter * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t tS = tS0 + q * kTN, tO = tO0 + q * D;
+    if (warp < 4) publish_block_info(p, sd, ctl.bi, bf, pr == 0 && h == 0);
+    softmax_bar_sync();
+    const int r = (qt0 + q) * kBM + t;  // sequence-relative query row
+    const bool active = q < nq;
+    const RowInfo ri = row_info(sd, ctl.bi, r);
+    const RowMasks rm = row_masks(ri, ctl.bi, sd);
+    const float sl = p.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = active;
+    for (int j = 0; j < n_kt && ok; ++j) {
+      const bool masked = tile_needs_mask(sd, j * kTN);
+      const uint64_t vis0 = masked ? vis64(sd, j * kTN, rm) : ~0ull;
+      const uint64_t vis1 = masked ? vis64(sd, j * kTN + 64, rm) : ~0ull;
+      ok = !*abort_flag && mbar_wait(&ctl.s_full[q], j & 1);
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      tc_fence_after();
+      // pass 1: the row maximum over the tile's 128 keys
+      const float mt = masked ? tile_row_max<true>(tS + lane_off, vis0, vis1)
+                              : tile_row_max<false>(tS + lane_off, vis0, vis1);
+      // Raise the reference maximum on the first finite value, or when the tile maximum
+      // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
+      float m_new = m_run;
+      if (m_run == -INFINITY) m_new = mt;
+      else if ((mt - m_run) * sl > kRescaleLog2) m_new = mt;
+      const bool rescale = (m_new != m_run) && (m_run != -INFINITY);
+      const float alpha = rescale ? ex2_approx((m_run - m_new) * sl) : 1.f;
+      const float mL = (m_new == -INFINITY) ? 0.f : m_new * sl;
+      // PV_q(j - 1) completed before S_q(j) was issued: O_q may be rescaled right away.
+      if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + lane_off + 32 * c, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          tmem_st32(tO + lane_off + 32 * c, o);
+        }
+      }
+      // pass 2: P over the first 64 columns of S_q(j), and the row sum
+      const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
+      uint64_t acc[4] = {0, 0, 0, 0};  // bit pattern 0 = +0.0f
+      if (masked) tile_row_exp<true>(tS + lane_off, vis0, vis1, sl2, nmL2, acc);
+      else tile_row_exp<false>(tS + lane_off, vis0, vis1, sl2, nmL2, acc);
+      float a0, a1, b0, b1;
+      f2_unpack(f2_add(acc[0], acc[1]), a0, a1);
+      f2_unpack(f2_add(acc[2], acc[3]), b0, b1);
+      l_run = l_run * alpha + ((a0 + a1) + (b0 + b1));
+      m_run = m_new;
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.p_full[q]);
+    }
+    if (active) {
+      if (ok) ok = mbar_wait(&ctl.o_full[q], 0);
+      const bool wok = __all_sync(0xffffffffu, ok);
+      if (!wok && lane == 0) flag_timeout(p, ctl);
+      // O row / row sum -> bf16 into the tile's query buffer (no MMA reads it once o_full
+      // has completed), 16-byte chunks XOR-swizzled by row; then the tile's 128 threads
+      // store whole rows, coalesced.
+      constexpr int kChunks = D / 8;  // 16-byte chunks per output row
+      uint4* stage = reinterpret_cast<uint4*>(sQ + q * kTileBytes);
+      if (wok) {
+        tc_fence_after();
+        const float inv_l = 1.0f / l_run;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t rr[32];
+          tmem_ld32(tO + lane_off + 32 * c, rr);
+          tmem_wait_ld();
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 u;
+            u.x = pack_bf16x2(__uint_as_float(rr[8 * v + 0]) * inv_l, __uint_as_float(rr[8 * v + 1]) * inv_l);
+            u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
+            u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
+            u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
+            const int chunk = c * 4 + v;
+            stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
+          }
+        }
+      }
+      ctl.store_row[q][t] = (wok && ri.store && r < rows_seq) ? 1 : 0;
+      tile_bar_sync(q);
+      if (!*abort_flag) {
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o);
+        const int rbase = row0 + (qt0 + q) * kBM;
+#pragma unroll 4
+        for (int idx = t; idx < kBM * kChunks; idx += kBM) {
+          const int row = idx / kChunks, chunk = idx % kChunks;
+          if (ctl.store_row[q][row]) {
+            const uint4 u = stage[row * kChunks + (chunk ^ (row & (kChunks - 1)))];
+            uint4* dst = reinterpret_cast<uint4*>(
+                out + (static_cast<size_t>(rbase + row) * p.hq + h) * D);
+            dst[chunk] = u;
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWMma) {
+    tc_fence_after();
+    tmem_dealloc<kTmemCols>(ctl.tmem_base);
+  }
+}
+
 // ---------------------------------------------------------------- fp32 CUDA-core path
 template <int D>
 __global__ void __launch_bounds__(128) attn_simt(const __grid_constant__ AttnParams p) {
@@ -812,17 +1226,37 @@ cudaError_t ensure_smem_attr(F* kernel, size_t bytes, std::atomic<uint64_t>& don
   return e;
 }
 
+// attn_tc2 (two query tiles per CTA) halves the K/V traffic per query row and the number
+// of CTAs, which wins while per-CTA setup and launch waves dominate; on long sequences the
+// steady-state tile rate of attn_tc1 (query operand in TMEM, S from TMEM x shared memory)
+// wins. The switch point is the longest sequence's number of 128-key tiles.
+constexpr int kTc2MaxKeyTiles = 24;
+
 template <int D>
 cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
-  static std::atomic<uint64_t> attr_done{0};
-  CUtensorMap mk, mv;
+  static std::atomic<uint64_t> attr1_done{0}, attr2_done{0};
+  int max_kt = 0;
+  for (int s = 0; s < p.num_seqs; ++s)
+    max_kt = std::max(max_kt, (p.seq[s].n_orig + p.seq[s].slen + kTN - 1) / kTN);
+  CUtensorMap mq, mk, mv;
   if (!make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
       !make_map(&mv, p.v, p.hkv, D, p.total_rows, kTN))
     return cudaErrorInvalidValue;
-  const size_t smem = tc_smem_bytes<D>();
-  cudaError_t e = ensure_smem_attr(attn_tc<D>, smem, attr_done);
-  if (e != cudaSuccess) return e;
-  attn_tc<D><<<p.total_work, kTcThreads, smem, stream>>>(p, mk, mv);
+  // DARD_ATTN_TC=1 or 2 forces one kernel (tests and tuning); anything else: by length
+  const char* force = std::getenv("DARD_ATTN_TC");
+  const int forced = force ? std::atoi(force) : 0;
+  if (forced == 2 || (forced != 1 && max_kt <= kTc2MaxKeyTiles)) {
+    if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM)) return cudaErrorInvalidValue;
+    const size_t smem = tc2_smem_bytes<D>();
+    cudaError_t e = ensure_smem_attr(attn_tc2<D>, smem, attr2_done);
+    if (e != cudaSuccess) return e;
+    attn_tc2<D><<<p.total_pairs, kTc2Threads, smem, stream>>>(p, mq, mk, mv);
+  } else {
+    const size_t smem = tc1_smem_bytes<D>();
+    cudaError_t e = ensure_smem_attr(attn_tc1<D>, smem, attr1_done);
+    if (e != cudaSuccess) return e;
+    attn_tc1<D><<<p.total_work, kTc1Threads, smem, stream>>>(p, mk, mv);
+  }
   return cudaGetLastError();
 }
 

@@ -39,8 +39,10 @@ struct AttnParams {
   int32_t total_work;        // number of (sequence, q-tile, head) work items
   // Work items in longest-first order: sequence order[r] owns items
   // [work_prefix[r], work_prefix[r+1]), laid out q-tile major, head minor.
+  int32_t total_pairs;       // number of (sequence, pair of q-tiles, head) work items
   int32_t order[DARD_MAX_SEQS];
   int32_t work_prefix[DARD_MAX_SEQS + 1];
+  int32_t pair_prefix[DARD_MAX_SEQS + 1];  // the same over pairs of q-tiles
   SeqDesc seq[DARD_MAX_SEQS];
 };
 

@@ -11,6 +11,13 @@ from . import parity as P
 pytestmark = pytest.mark.gpu
 
 
+@pytest.fixture(params=["1", "2"])
+def tc(request, monkeypatch):
+    """Runs the test once per tensor-core kernel (one or two query tiles per CTA)."""
+    monkeypatch.setenv("DARD_ATTN_TC", request.param)
+    return request.param
+
+
 def _attend(wl, layer=0, scale=0.0):
     ds = DeviceStep(wl, layers=[layer], scoring=False)
     o = ds.attention(0, scale=scale)
@@ -24,7 +31,7 @@ def _attend(wl, layer=0, scale=0.0):
     ("gqa", "paper", 192), ("gqa", "candidates", 192),
     ("ragged", "paper", 48), ("mm", "paper", 64),
 ])
-def test_attention_configs(name, layout, sample):
+def test_attention_configs(name, layout, sample, tc):
     wl = W.make(name, layout=layout, scoring=False, layers=2 if name == "mm" else None)
     layers = [0, 1] if name == "mm" else [0]
     for li in layers:
@@ -44,7 +51,7 @@ def _probe_tol(wl):
 
 @pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("layout", ["paper", "candidates"])
-def test_mask_probe_every_key(d, layout):
+def test_mask_probe_every_key(d, layout, tc):
     """Uniform attention (Q = 0) exposes every key selection of the in-kernel mask."""
     specs = [dict(n_orig=200, block_start=100, block_len=64, fractions=(0.3, 0.4, 0.3),
                   shadow=layout),
@@ -59,7 +66,7 @@ def test_mask_probe_every_key(d, layout):
     assert mx <= _probe_tol(wl)
 
 
-def test_mask_probe_confidence_ties():
+def test_mask_probe_confidence_ties(tc):
     """Equal c_{t-1} among C tokens attend each other both ways (Eq. 3 uses <=)."""
     B = 48
     st = np.array([1] * 24 + [0] * 12 + [2] * 12, dtype=np.uint8)
@@ -75,7 +82,7 @@ def test_mask_probe_confidence_ties():
 
 
 @pytest.mark.parametrize("states", ["M", "C", "U"])
-def test_mask_probe_uniform_states(states):
+def test_mask_probe_uniform_states(states, tc):
     code = {"M": 0, "C": 1, "U": 2}[states]
     specs = [dict(n_orig=256, block_start=128, state=np.full(64, code, np.uint8))]
     wl = W.custom(specs, 2, 1, 128, probe=True, seed=code)
@@ -85,7 +92,7 @@ def test_mask_probe_uniform_states(states):
 
 
 @pytest.mark.parametrize("case", range(12))
-def test_attention_random_shapes(case):
+def test_attention_random_shapes(case, tc):
     """Seeded random ragged batches: odd lengths, blocks at the start / end, S = 0,
     B = 1..128, grouped heads, larger scores (scale up to 1) to exercise the O rescale."""
     rng = np.random.default_rng(100 + case)
@@ -112,7 +119,7 @@ def test_attention_random_shapes(case):
     assert mx <= P.att_tol(wl) and mean <= P.ATT_MEAN_ABS
 
 
-def test_attention_bad_shadow_rows_flagged():
+def test_attention_bad_shadow_rows_flagged(tc):
     """shadow_src outside the block or repeated: status bit, other rows still correct."""
     specs = [dict(n_orig=128, block_start=32, block_len=16, fractions=(0.4, 0.3, 0.3),
                   shadow=np.array([32, 33, 34, 34, 90, 35], np.int32))]
