@@ -116,6 +116,17 @@ def peaks():
     return 6800.0, 1900.0, "fallback"
 
 
+def attention_kernel(wl) -> str:
+    """The tensor-core attention kernel the library runs for this batch: two query tiles per
+    CTA while the longest sequence has at most 24 tiles of 128 keys, else one (or the one
+    DARD_ATTN_TC forces)."""
+    forced = os.environ.get("DARD_ATTN_TC", "")
+    if forced in ("1", "2"):
+        return f"attn_tc{forced}"
+    max_kt = max((s.rows + 127) // 128 for s in wl.seqs)
+    return "attn_tc2" if max_kt <= 24 else "attn_tc1"
+
+
 def traffic_for(kernel: str, source: str, per_launch_units: float):
     """DRAM bytes per launch from profiles/traffic.txt, if recorded for this source hash."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
@@ -348,6 +359,7 @@ def run_ours(args, rank: int, world: int):
     if rank != 0:
         return
     hbm, bf16, peak_kind = peaks()
+    attn_kernel = attention_kernel(wl)
     flops = W.attention_flops(wl)
     sbytes = W.scoring_bytes(wl)
     att_tflops = flops / (attn_us * 1e-6) / 1e12
@@ -360,10 +372,10 @@ def run_ours(args, rank: int, world: int):
         "config": {"workload": WORKLOAD_DESC, "layout": args.layout,
                    "l2": f"{NSETS} rotating input sets (~675 MB) > 4x L2",
                    "parallelism": f"replicas x{world}", "timing": "CUDA-graph replays"},
-        "roofline": {"bound": "tensor", "kernel": "attn_tc<128>", "achieved": att_tflops,
+        "roofline": {"bound": "tensor", "kernel": f"{attn_kernel}<128>", "achieved": att_tflops,
                      "peak": bf16, "unit": "TFLOP/s", "frac": att_tflops / bf16,
                      "peak_kind": f"{peak_kind} bf16 burst",
-                     "traffic": traffic_for("attn_tc", "paper_2608_26574_gb300/csrc/dard_attention.cu", 1.0),
+                     "traffic": traffic_for(attn_kernel, "paper_2608_26574_gb300/csrc/dard_attention.cu", 1.0),
                      "algorithmic_flops_per_launch": flops},
         "kernels": {"attention_us": attn_us, "attention_tflops": att_tflops,
                     "attention_frac_bf16": att_tflops / bf16, "scoring_us": score_us,

@@ -71,6 +71,7 @@ struct ScoreParams {
 
 constexpr int kScoreThreads = 256;
 constexpr int kScoreMaxSplit = 16;  // CTAs per row = thread-block cluster size
+constexpr int kScoreCtasPerSm = 12;  // target CTAs per SM when choosing the split
 
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs);
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,

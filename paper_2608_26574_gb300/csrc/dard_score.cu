@@ -16,9 +16,9 @@
 // (deterministic) and writes the row's outputs. Pass 2 is launched as a programmatic
 // dependent of pass 1: its CTAs load their logits while pass 1 finishes and only then
 // wait for pass 1's results.
+#include <atomic>
 #include <cfloat>
 #include <climits>
-#include <atomic>
 #include <cmath>
 #include <cstdio>
 
@@ -420,20 +420,47 @@ size_t score_workspace_bytes(int32_t rows, int32_t num_seqs) {
   return (static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
 }
 
+namespace {
+
+// Number of SMs of the current device (looked up once per device).
+int sm_count() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (n <= 0) {
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cache[dev].store(n, std::memory_order_relaxed);
+  }
+  return n;
+}
+
+// CTAs per row: few rows spread over up to kScoreMaxSplit CTAs so that the call still has
+// about kScoreCtasPerSm CTAs per SM in flight; many rows get one or a few CTAs each, every
+// CTA then streaming more rounds of its row (fewer merges, deeper per-CTA pipelines).
+int split_cap(int rows) {
+  const long long want = (static_cast<long long>(kScoreCtasPerSm) * sm_count() + rows - 1) /
+                         std::max(rows, 1);
+  return static_cast<int>(std::max(1ll, std::min<long long>(kScoreMaxSplit, want)));
+}
+
+}  // namespace
+
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
                          char* err, size_t err_len) {
   const bool bf16 = a.dtype == DARD_BF16;
   const int W = bf16 ? 8 : 4;
-  // One round = 256 threads x 4 vectors; a row spreads over at most kScoreMaxSplit CTAs
-  // (one cluster), each taking `rounds` rounds.
+  // One round = 256 threads x 4 vectors; a row spreads over at most split_cap() CTAs (one
+  // cluster), each taking `rounds` rounds.
   const int per_round = kScoreThreads * 4 * W;
   const int rounds_total = (p.vocab + per_round - 1) / per_round;
-  const int rounds = (rounds_total + kScoreMaxSplit - 1) / kScoreMaxSplit;
+  const int cap = split_cap(p.rows);
+  const int rounds = (rounds_total + cap - 1) / cap;
   p.chunk = per_round * rounds;
   p.nsplit = (p.vocab + p.chunk - 1) / p.chunk;
 
   char* ws = static_cast<char*>(a.workspace);
-  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
   p.pd_flag = reinterpret_cast<uint8_t*>(ws);
   p.log2_lambda = static_cast<float>(std::log2(static_cast<double>(p.lambda)));
 
