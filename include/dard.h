@@ -110,6 +110,11 @@ typedef struct {
                                 in [b0_i, b0_i + B_i), distinct within a sequence          */
   float scale;               /* softmax scale; 0 means 1/sqrt(head_dim)                    */
   uint32_t* status;          /* optional device word, DARD_STATUS_* bits OR-ed in          */
+  const int32_t* query_start;/* optional host [num_seqs] q_i in 0 .. N_i + S_i: only rows
+                                q_i .. N_i + S_i - 1 of sequence i are queries (prefix
+                                caching: the prompt's outputs are not recomputed, its
+                                K/V rows still serve as keys); rows before q_i of o are
+                                left untouched. NULL means 0 for every sequence.           */
 } dard_attn_args;
 
 /* Rows are total_rows = sum_i (N_i + S_i). q, k, v, o must be 16-byte aligned; with dtype

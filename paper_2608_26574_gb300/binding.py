@@ -31,7 +31,8 @@ class AttnArgs(ctypes.Structure):
                 ("num_seqs", ctypes.c_int32), ("n_orig", _I32P), ("block_start", _I32P),
                 ("block_len", _I32P), ("shadow_len", _I32P), ("state", ctypes.c_void_p),
                 ("prev_conf", ctypes.c_void_p), ("shadow_src", ctypes.c_void_p),
-                ("scale", ctypes.c_float), ("status", ctypes.c_void_p)]
+                ("scale", ctypes.c_float), ("status", ctypes.c_void_p),
+                ("query_start", _I32P)]
 
 
 class ScoreArgs(ctypes.Structure):
@@ -132,9 +133,12 @@ def _dtype_code(t) -> int:
 
 
 def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, state,
-                        prev_conf, shadow_src, scale: float = 0.0, status=None, stream=None):
-    """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d] on the device."""
+                        prev_conf, shadow_src, scale: float = 0.0, status=None, stream=None,
+                        query_start=None):
+    """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d] on the device.
+    ``query_start`` (per sequence, optional): first query row; earlier rows are keys only."""
     n_orig, block_start = _host_i32(n_orig), _host_i32(block_start)
+    qs = _host_i32(query_start) if query_start is not None else None
     block_len, shadow_len = _host_i32(block_len), _host_i32(shadow_len)
     a = AttnArgs()
     a.q, a.k, a.v, a.o = _ptr(q), _ptr(k), _ptr(v), _ptr(o)
@@ -148,6 +152,7 @@ def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, 
     a.state, a.prev_conf, a.shadow_src = _ptr(state), _ptr(prev_conf), _ptr(shadow_src)
     a.scale = scale
     a.status = _ptr(status)
+    a.query_start = qs.ctypes.data_as(_I32P) if qs is not None else None
     _check(lib().dard_step_attention(ctypes.byref(a), _stream(stream)), "dard_step_attention")
 
 

@@ -86,6 +86,9 @@ dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
     if (b0 < 0 || static_cast<long long>(b0) + B > n)
       return fail(DARD_ERR_SHAPE, "seq %d: block [%d, %d) outside [0, %d)", s, b0, b0 + B, n);
     if (S < 0 || S > B) return fail(DARD_ERR_SHAPE, "seq %d: shadow_len %d outside 0..%d", s, S, B);
+    const int qs = a->query_start ? a->query_start[s] : 0;
+    if (qs < 0 || qs > n + S)
+      return fail(DARD_ERR_SHAPE, "seq %d: query_start %d outside 0..%d", s, qs, n + S);
     SeqDesc& d = p.seq[s];
     d.row_base = static_cast<int32_t>(rows);
     d.n_orig = n;
@@ -94,7 +97,8 @@ dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
     d.slen = S;
     d.blk_off = static_cast<int32_t>(blk);
     d.sh_off = static_cast<int32_t>(sh);
-    d.n_qtiles = (n + S + 127) / 128;
+    d.q_start = qs;
+    d.n_qtiles = (n + S - qs + 127) / 128;
     cost[s] = static_cast<long long>(n) + S;
     rows += n + S;
     blk += B;
@@ -139,6 +143,7 @@ dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
   p.num_seqs = a->num_seqs;
   p.scale = a->scale > 0.f ? a->scale : 1.0f / std::sqrt(static_cast<float>(a->head_dim));
   p.scale_log2 = p.scale * 1.4426950408889634f;
+  if (p.total_work == 0) return DARD_OK;  // no query rows (every query_start at the end)
   return launch_attention(*a, p, static_cast<cudaStream_t>(stream), g_err, sizeof(g_err));
 }
 

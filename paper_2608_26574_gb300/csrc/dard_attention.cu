@@ -409,7 +409,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
   const SeqDesc sd = p.seq[seq];
   const int rows_seq = sd.n_orig + sd.slen;
   const int n_kt = (rows_seq + kTN - 1) / kTN;
-  const int q0 = qt * kBM;
+  const int q0 = sd.q_start + qt * kBM;  // first (sequence-relative) query row of the tile
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -911,7 +911,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
 #pragma unroll
       for (int s = 0; s < kSub; ++s)
         tma_load_2d(sQ + q * kTileBytes + s * kKSub, &tmq, &ctl.q_full, h * D + s * 64,
-                    row0 + (qt0 + q) * kBM);
+                    row0 + sd.q_start + (qt0 + q) * kBM);
     }
     for (int j = 0; j < kNK && j < n_kt; ++j) load_kv(j, true);
     for (int j = 0; j < kNV && j < n_kt; ++j) load_kv(j, false);
@@ -1023,7 +1023,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     const uint32_t tS = tS0 + q * kTN, tO = tO0 + q * D;
     if (warp < 4) publish_block_info(p, sd, ctl.bi, bf, pr == 0 && h == 0);
     softmax_bar_sync();
-    const int r = (qt0 + q) * kBM + t;  // sequence-relative query row
+    const int r = sd.q_start + (qt0 + q) * kBM + t;  // sequence-relative query row
     const bool active = q < nq;
     const RowInfo ri = row_info(sd, ctl.bi, r);
     const RowMasks rm = row_masks(ri, ctl.bi, sd);
@@ -1108,7 +1108,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       tile_bar_sync(q);
       if (!*abort_flag) {
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o);
-        const int rbase = row0 + (qt0 + q) * kBM;
+        const int rbase = row0 + sd.q_start + (qt0 + q) * kBM;
 #pragma unroll 4
         for (int idx = t; idx < kBM * kChunks; idx += kBM) {
           const int row = idx / kChunks, chunk = idx % kChunks;
@@ -1148,7 +1148,7 @@ __global__ void __launch_bounds__(128) attn_simt(const __grid_constant__ AttnPar
   float* O = static_cast<float*>(p.o);
   const float scale = p.scale;
   for (int rr = 0; rr < 32; ++rr) {
-    const int r = qt * kBM + warp * 32 + rr;
+    const int r = sd.q_start + qt * kBM + warp * 32 + rr;
     if (r >= rows_seq) break;
     const RowInfo q = row_info(sd, bi, r);
     if (!q.store) continue;

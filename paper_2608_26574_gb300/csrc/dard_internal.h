@@ -20,7 +20,8 @@ struct SeqDesc {
   int32_t slen;       // S
   int32_t blk_off;    // offset of the block in state / prev_conf
   int32_t sh_off;     // offset of the shadow rows in shadow_src
-  int32_t n_qtiles;   // ceil((N + S) / 128)
+  int32_t q_start;    // first query row (rows before it are keys only)
+  int32_t n_qtiles;   // ceil((N + S - q_start) / 128)
 };
 
 struct AttnParams {

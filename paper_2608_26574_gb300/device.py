@@ -30,6 +30,8 @@ class DeviceStep:
         self.block_start = np.array([s.block_start for s in wl.seqs], dtype=np.int32)
         self.block_len = np.array([s.block_len for s in wl.seqs], dtype=np.int32)
         self.shadow_len = np.array([s.n_shadow for s in wl.seqs], dtype=np.int32)
+        qs = np.array([s.query_start for s in wl.seqs], dtype=np.int32)
+        self.query_start = qs if qs.any() else None
         dev = self.device
         self.state = torch.from_numpy(wl.state_all()).to(dev)
         self.prev_conf = torch.from_numpy(wl.prev_conf_all()).to(dev)
@@ -69,7 +71,8 @@ class DeviceStep:
         q, k, v, o = self.layers[layer]
         B.dard_step_attention(q, k, v, o if out is None else out, self.n_orig, self.block_start,
                               self.block_len, self.shadow_len, self.state, self.prev_conf,
-                              self.shadow_src, scale=scale, status=self.status, stream=stream)
+                              self.shadow_src, scale=scale, status=self.status, stream=stream,
+                              query_start=self.query_start)
         return o if out is None else out
 
     def score(self, stream=None, w_out=True, counts=True, state_in=None):

@@ -68,6 +68,8 @@ class Seq:
     state: np.ndarray       # uint8 [B]
     prev_conf: np.ndarray   # float32 [B]
     shadow_src: np.ndarray  # int32 [S]
+    prompt: int = 0         # prompt length P0 (positions 0 .. P0-1)
+    query_start: int = 0    # first query row (prefix caching: P0; 0 = every row is a query)
 
     @property
     def block_len(self) -> int:
@@ -180,9 +182,12 @@ def _logits(rng, nrows, vocab, std, dtype, mode, plant_frac, plant_height):
 
 
 def make(name: str, layout: str = "paper", logits: str = "literal", attention: bool = True,
-         scoring: bool = True, layers: int | None = None, seed: int | None = None) -> Workload:
+         scoring: bool = True, layers: int | None = None, seed: int | None = None,
+         prefix: bool = False) -> Workload:
     """Build one named workload. ``logits``: "literal" (the stated distribution and planted
-    peaks), "spanning" (planted confidences spread across the thresholds) or "plain"."""
+    peaks), "spanning" (planted confidences spread across the thresholds) or "plain".
+    ``prefix``: the prefix-cached variant, whose queries start after the prompt (the same
+    inputs; only which rows are queries changes)."""
     if seed is None:
         seed = SEED_BASE + CONFIG_INDEX[name]
     rng = np.random.default_rng(np.random.PCG64(seed))
@@ -191,21 +196,21 @@ def make(name: str, layout: str = "paper", logits: str = "literal", attention: b
 
     if name == "tiny":
         st, cf = _draw_states(rng, 32, (0.4, 0.3, 0.3), tau_c, tau_u)
-        seqs = [Seq(64, 32, st, cf, _shadow(st, 32, layout))]
+        seqs = [Seq(64, 32, st, cf, _shadow(st, 32, layout), prompt=32)]
         wl = Workload(name, "f32", 4, 4, 64, 1024, seqs, tau_c, tau_u)
         std_fn = lambda rows: np.ones(rows)  # noqa: E731
         lspec = (2.0, 0.5, 6.0)
     elif name == "8b":
         b0 = 512 + 3 * 32
         st, cf = _draw_states(rng, 32, (0.5, 0.25, 0.25), tau_c, tau_u)
-        seqs = [Seq(512 + 256, b0, st, cf, _shadow(st, b0, layout))]
+        seqs = [Seq(512 + 256, b0, st, cf, _shadow(st, b0, layout), prompt=512)]
         wl = Workload(name, "bf16", 32, 32, 128, 126464, seqs, tau_c, tau_u)
         std_fn = lambda rows: np.full(rows, isd)  # noqa: E731
         lspec = (3.0, 0.4, 6.0)
     elif name == "gqa":
         b0 = 4096 + 8 * 64
         st, cf = _draw_states(rng, 64, (0.3, 0.4, 0.3), tau_c, tau_u)
-        seqs = [Seq(4096 + 1024, b0, st, cf, _shadow(st, b0, layout))]
+        seqs = [Seq(4096 + 1024, b0, st, cf, _shadow(st, b0, layout), prompt=4096)]
         wl = Workload(name, "bf16", 28, 4, 128, 152064, seqs, tau_c, tau_u)
         std_fn = lambda rows: np.full(rows, isd)  # noqa: E731
         lspec = (3.0, 0.0, 0.0)
@@ -217,7 +222,7 @@ def make(name: str, layout: str = "paper", logits: str = "literal", attention: b
             fm = float(rng.uniform(0.2, 0.8))
             st, cf = _draw_states(rng, 32, (fm, (1 - fm) / 2, (1 - fm) / 2), tau_c, tau_u)
             b0 = p0 + 32 * idx
-            seqs.append(Seq(p0 + 256, b0, st, cf, _shadow(st, b0, layout)))
+            seqs.append(Seq(p0 + 256, b0, st, cf, _shadow(st, b0, layout), prompt=p0))
         wl = Workload(name, "bf16", 32, 32, 128, 126464, seqs, tau_c, tau_u)
         std_fn = lambda rows: np.full(rows, isd)  # noqa: E731
         lspec = (3.0, 0.4, 6.0)
@@ -226,7 +231,7 @@ def make(name: str, layout: str = "paper", logits: str = "literal", attention: b
         seqs = []
         for _ in range(8):
             st, cf = _draw_states(rng, 32, (0.2, 0.6, 0.2), tau_c, tau_u)
-            seqs.append(Seq(704 + 512, b0, st, cf, _shadow(st, b0, layout)))
+            seqs.append(Seq(704 + 512, b0, st, cf, _shadow(st, b0, layout), prompt=704))
         wl = Workload(name, "bf16", 32, 32, 128, 126464, seqs, tau_c, tau_u)
         wl.layers = 32 if layers is None else layers
 
@@ -241,6 +246,9 @@ def make(name: str, layout: str = "paper", logits: str = "literal", attention: b
     else:
         raise ValueError(name)
 
+    if prefix:
+        for sq in wl.seqs:
+            sq.query_start = sq.prompt
     if attention:
         for _ in range(wl.layers):
             q, k, v = _qkv(rng, wl.seqs, wl.hq, wl.hkv, wl.head_dim, wl.dtype, std_fn)
@@ -258,7 +266,8 @@ def make(name: str, layout: str = "paper", logits: str = "literal", attention: b
 def attention_flops(wl: Workload) -> float:
     """Algorithmic attention FLOPs of one layer: every query row attends exactly N keys
     (one copy per original position), QK^T and PV each 2*d FLOPs per (row, key, head)."""
-    return float(sum(4.0 * wl.head_dim * s.rows * s.n_orig * wl.hq for s in wl.seqs))
+    return float(sum(4.0 * wl.head_dim * (s.rows - s.query_start) * s.n_orig * wl.hq
+                     for s in wl.seqs))
 
 
 def scoring_bytes(wl: Workload) -> float:
@@ -297,7 +306,8 @@ def custom(specs, hq: int, hkv: int, head_dim: int, dtype: str = "bf16", vocab: 
         shadow = sp.get("shadow", "paper")
         src = _shadow(st, sp["block_start"], shadow) if isinstance(shadow, str) else \
             np.asarray(shadow, dtype=np.int32)
-        seqs.append(Seq(sp["n_orig"], sp["block_start"], st, cf, src))
+        seqs.append(Seq(sp["n_orig"], sp["block_start"], st, cf, src,
+                        query_start=int(sp.get("query_start", 0))))
     wl = Workload("custom", dtype, hq, hkv, head_dim, vocab, seqs, tau_c, tau_u)
     std = (1.0 / math.sqrt(head_dim)) if qkv_std is None else qkv_std
     rows = wl.total_rows

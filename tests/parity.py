@@ -48,15 +48,18 @@ def compare_attention(wl, layer, o_host, sample=None, scale=None, rng=None):
     offs = wl.row_offsets()
     errs, n = [], 0
     for si, s in enumerate(wl.seqs):
-        R = s.rows
-        if sample is None or sample >= R:
-            rows = np.arange(R)
+        R, q0 = s.rows, s.query_start  # rows before q0 are keys only (prefix caching)
+        if q0 >= R:
+            continue
+        if sample is None or sample >= R - q0:
+            rows = np.arange(q0, R)
         else:
             rng = rng or np.random.default_rng(0)
             must = np.concatenate([np.arange(s.block_start, s.block_start + s.block_len),
-                                   np.arange(s.n_orig, R), [0, R - 1]])
-            extra = rng.choice(R, size=sample, replace=False)
+                                   np.arange(s.n_orig, R), [q0, R - 1]])
+            extra = q0 + rng.choice(R - q0, size=sample, replace=False)
             rows = np.unique(np.concatenate([must, extra]).astype(np.int64))
+            rows = rows[rows >= q0]
         ref = oracle_attention(wl, layer, si, rows=rows, scale=scale)
         got = o_host[offs[si] + rows].astype(np.float64)
         errs.append(np.abs(got - ref).reshape(len(rows), -1))

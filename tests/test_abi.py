@@ -57,6 +57,9 @@ def _attn_args(**kw):
     a.q = a.k = a.v = a.o = 0x10000
     a.dtype, a.hq, a.hkv, a.head_dim, a.num_seqs = B.DARD_BF16, 4, 4, 64, 1
     keep = {"n": kw.pop("n", n), "b0": kw.pop("b0", b0), "bl": kw.pop("bl", bl), "sl": kw.pop("sl", sl)}
+    if "qs" in kw:
+        keep["qs"] = kw.pop("qs")
+        a.query_start = keep["qs"].ctypes.data_as(B._I32P)
     a.n_orig = keep["n"].ctypes.data_as(B._I32P)
     a.block_start = keep["b0"].ctypes.data_as(B._I32P)
     a.block_len = keep["bl"].ctypes.data_as(B._I32P)
@@ -76,6 +79,7 @@ def _attn_args(**kw):
     ({"n": np.array([0], np.int32)}, 2), ({"bl": np.array([129], np.int32)}, 2),
     ({"b0": np.array([40], np.int32)}, 2), ({"sl": np.array([33], np.int32)}, 2),
     ({"b0": np.array([-1], np.int32)}, 2),
+    ({"qs": np.array([97], np.int32)}, 2), ({"qs": np.array([-1], np.int32)}, 2),
 ])
 def test_attention_validation(lib, change, code):
     a, keep = _attn_args(**change)

@@ -134,3 +134,57 @@ def test_attention_bad_shadow_rows_flagged(tc):
     good.q[0], good.k[0], good.v[0] = wl.q[0][keep], wl.k[0][keep], wl.v[0][keep]
     ref = P.oracle_attention(good, 0, 0)
     np.testing.assert_allclose(o[keep], ref, atol=P.ATT_MAX_ABS)
+
+
+def _sentinel_out(ds):
+    q = ds.layers[0][0]
+    return torch.full_like(q, 7.0)
+
+
+@pytest.mark.parametrize("name,sample", [("tiny", None), ("8b", None), ("gqa", 192),
+                                         ("ragged", 48), ("mm", 64)])
+def test_attention_prefix_cached(name, sample, tc):
+    """Prefix caching (queries from the prompt's end on): the kept rows match the oracle,
+    and the output rows of the cached prompt are left untouched."""
+    wl = W.make(name, prefix=True, scoring=False, layers=1 if name == "mm" else None)
+    ds = DeviceStep(wl, layers=[0], scoring=False)
+    out = _sentinel_out(ds)
+    ds.attention(0, out=out)
+    torch.cuda.synchronize()
+    o = out.float().cpu().numpy()
+    mx, mean, n = P.compare_attention(wl, 0, o, sample=sample)
+    assert mx <= P.att_tol(wl, 0) and mean <= P.ATT_MEAN_ABS
+    offs = wl.row_offsets()
+    for si, s in enumerate(wl.seqs):
+        assert s.query_start == s.prompt > 0
+        assert np.all(o[offs[si]:offs[si] + s.query_start] == 7.0)
+    assert int(ds.status.item()) == 0
+
+
+@pytest.mark.parametrize("case", range(6))
+def test_attention_random_query_start(case, tc):
+    """Random per-sequence query starts, including none (all rows) and the end (no rows)."""
+    rng = np.random.default_rng(700 + case)
+    specs = []
+    for si in range(int(rng.integers(1, 5))):
+        n = int(rng.integers(1, 600))
+        B = int(rng.integers(0, min(n, 128) + 1))
+        b0 = int(rng.integers(0, n - B + 1))
+        sp = dict(n_orig=n, block_start=b0, block_len=B, fractions=tuple(rng.dirichlet([1, 1, 1])))
+        rows = n + B
+        sp["query_start"] = int(rng.choice([0, rows, int(rng.integers(0, rows + 1))]))
+        specs.append(sp)
+    hkv = int(rng.choice([1, 2]))
+    d = int(rng.choice([64, 128]))
+    wl = W.custom(specs, hkv * 2, hkv, d, seed=800 + case)
+    ds = DeviceStep(wl, layers=[0], scoring=False)
+    out = _sentinel_out(ds)
+    ds.attention(0, out=out)
+    torch.cuda.synchronize()
+    o = out.float().cpu().numpy()
+    if any(s.query_start < s.rows for s in wl.seqs):
+        mx, mean, n = P.compare_attention(wl, 0, o)
+        assert mx <= P.att_tol(wl) and mean <= P.ATT_MEAN_ABS
+    offs = wl.row_offsets()
+    for si, s in enumerate(wl.seqs):
+        assert np.all(o[offs[si]:offs[si] + s.query_start] == 7.0)
