@@ -116,15 +116,27 @@ def peaks():
     return 6800.0, 1900.0, "fallback"
 
 
-def attention_kernel(wl) -> str:
-    """The tensor-core attention kernel the library runs for this batch: two query tiles per
-    CTA while the longest sequence has at most 24 tiles of 128 keys, else one (or the one
-    DARD_ATTN_TC forces)."""
+def attention_kernel(wl, sms: int = 152) -> str:
+    """The tensor-core attention kernel the library picks for this batch (the same cost
+    model as the library's launcher), or the one DARD_ATTN_TC forces."""
     forced = os.environ.get("DARD_ATTN_TC", "")
     if forced in ("1", "2"):
         return f"attn_tc{forced}"
-    max_kt = max((s.rows + 127) // 128 for s in wl.seqs)
-    return "attn_tc2" if max_kt <= 24 else "attn_tc1"
+
+    def cycles(items):
+        total = sum(n * c for n, c in items)
+        ctas = sum(n for n, _ in items)
+        longest = max([c for n, c in items if n > 0] or [0.0])
+        return longest if ctas <= sms else total / sms + 0.5 * longest
+
+    one, two = [], []
+    for s in wl.seqs:
+        kt = (s.rows + 127) // 128
+        tiles = (s.rows - s.query_start + 127) // 128
+        one.append((tiles * wl.hq, 14700.0 + 1480.0 * kt))
+        two.append(((tiles // 2) * wl.hq, 13900.0 + 3770.0 * kt))
+        two.append(((tiles % 2) * wl.hq, 8800.0 + 3000.0 * kt))
+    return "attn_tc2" if cycles(two) < cycles(one) else "attn_tc1"
 
 
 def traffic_for(kernel: str, source: str, per_launch_units: float):

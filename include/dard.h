@@ -119,10 +119,10 @@ typedef struct {
 
 /* Rows are total_rows = sum_i (N_i + S_i). q, k, v, o must be 16-byte aligned; with dtype
  * BF16 a tensor-core kernel runs (head_dim 64 or 128), with F32 the CUDA-core kernel.
- * Of the two tensor-core kernels, the one with two 128-row query tiles per CTA serves
- * batches whose longest sequence has at most 24 tiles of 128 keys (N_i + S_i <= 3072), the
- * one with one query tile per CTA longer ones; the environment variable DARD_ATTN_TC=1 or 2
- * forces one of them (results agree within rounding).
+ * Of the two tensor-core kernels (one or two 128-row query tiles per CTA) the library
+ * picks the one a cost model of the batch (query tiles, key tiles, SM count) predicts to be
+ * faster; the environment variable DARD_ATTN_TC=1 or 2 forces one of them (results agree
+ * within rounding).
  * Errors: DARD_ERR_NULL, _SHAPE, _VALUE (scale < 0 or not finite), _UNSUPPORTED,
  * _ALIGN, _CUDA. */
 dard_status dard_step_attention(const dard_attn_args* args, void* stream /* cudaStream_t */);

@@ -1226,26 +1226,66 @@ cudaError_t ensure_smem_attr(F* kernel, size_t bytes, std::atomic<uint64_t>& don
   return e;
 }
 
-// attn_tc2 (two query tiles per CTA) halves the K/V traffic per query row and the number
-// of CTAs, which wins while per-CTA setup and launch waves dominate; on long sequences the
-// steady-state tile rate of attn_tc1 (query operand in TMEM, S from TMEM x shared memory)
-// wins. The switch point is the longest sequence's number of 128-key tiles.
-constexpr int kTc2MaxKeyTiles = 24;
+// Which tensor-core kernel: a cost model in SM cycles, fitted (least squares on the log of
+// the time) to CUDA-graph timings of both kernels on the full and prefix-cached variants
+// of four workload shapes on GB300, within 5 % of each. attn_tc1 costs about
+// 14700 + 1480 kt cycles per 128-row query tile (kt = tiles of 128 keys); attn_tc2 about
+// 13900 + 3770 kt per pair of tiles and 8800 + 3000 kt for a lone last tile. Work spreads
+// over the SMs one CTA each: a launch with no more CTAs than SMs takes its longest CTA, a
+// larger one about total / SMs plus half a CTA of tail. attn_tc2 wins when few waves and
+// per-CTA setup dominate (8B layer: one wave instead of 1.5), attn_tc1 on long sequences
+// and on small query counts (prefix caching).
+struct TcEstimate {
+  double total = 0, longest = 0;
+  long long ctas = 0;
+  void add(long long n, double cost) {
+    if (n <= 0) return;
+    total += static_cast<double>(n) * cost;
+    longest = std::max(longest, cost);
+    ctas += n;
+  }
+  double cycles(int sms) const {
+    return ctas <= sms ? longest : total / sms + 0.5 * longest;
+  }
+};
+
+bool prefer_tc2(const AttnParams& p, int sms) {
+  TcEstimate one, two;
+  for (int s = 0; s < p.num_seqs; ++s) {
+    const SeqDesc& sd = p.seq[s];
+    const double kt = (sd.n_orig + sd.slen + kTN - 1) / kTN;
+    const long long tiles = sd.n_qtiles, heads = p.hq;
+    one.add(tiles * heads, 14700.0 + 1480.0 * kt);
+    two.add((tiles / 2) * heads, 13900.0 + 3770.0 * kt);
+    two.add((tiles % 2) * heads, 8800.0 + 3000.0 * kt);
+  }
+  return two.cycles(sms) < one.cycles(sms);
+}
+
+int sm_count() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (n <= 0) {
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cache[dev].store(n, std::memory_order_relaxed);
+  }
+  return n;
+}
 
 template <int D>
 cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
   static std::atomic<uint64_t> attr1_done{0}, attr2_done{0};
-  int max_kt = 0;
-  for (int s = 0; s < p.num_seqs; ++s)
-    max_kt = std::max(max_kt, (p.seq[s].n_orig + p.seq[s].slen + kTN - 1) / kTN);
   CUtensorMap mq, mk, mv;
   if (!make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
       !make_map(&mv, p.v, p.hkv, D, p.total_rows, kTN))
     return cudaErrorInvalidValue;
-  // DARD_ATTN_TC=1 or 2 forces one kernel (tests and tuning); anything else: by length
+  // DARD_ATTN_TC=1 or 2 forces one kernel (tests and tuning); anything else: the model
   const char* force = std::getenv("DARD_ATTN_TC");
   const int forced = force ? std::atoi(force) : 0;
-  if (forced == 2 || (forced != 1 && max_kt <= kTc2MaxKeyTiles)) {
+  if (forced == 2 || (forced != 1 && prefer_tc2(p, sm_count()))) {
     if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM)) return cudaErrorInvalidValue;
     const size_t smem = tc2_smem_bytes<D>();
     cudaError_t e = ensure_smem_attr(attn_tc2<D>, smem, attr2_done);
