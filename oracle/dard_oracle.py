@@ -31,7 +31,12 @@ Readings of points the paper leaves open (each is listed in the design doc):
   R6  a scored row is invalid when its softmax normaliser is not finite or is zero
       (NaN, +inf, or all -inf logits): confidence 0, token -1, state M;
   R7  a state byte above 2 is treated as M;
-  R8  the attention scale is 1/sqrt(head_dim) unless given.
+  R8  the attention scale is 1/sqrt(head_dim) unless given;
+  R9  p_cur, reported beside c, is the probability the scored distribution (shadow logits
+      for C and U positions, mixed logits for M positions) gives to the token currently at
+      the position; 0 for a token outside the vocabulary or an invalid row;
+  R10 the token update that closes a step of Algorithm 1: positions that end the step in
+      M hold the mask token again, every other position holds its new prediction x^.
 
 Parity pins: every function here is pinned by ``tests/test_oracle_pins.py`` except where
 a docstring says "parity unpinned".
@@ -240,6 +245,26 @@ def confidence(logits_row: np.ndarray) -> tuple[float, int, bool]:
     return float(1.0 / z), token, True
 
 
+def token_probability(logits_row: np.ndarray, tok: int) -> float:
+    """R9: softmax(logits)[tok] in float64, i.e. exp(l_tok - max) / sum exp(l - max).
+
+    0.0 for tok outside [0, V) or an invalid row (R6).
+    """
+    x = logits_row.astype(np.float64)
+    if not (0 <= tok < len(x)):
+        return 0.0
+    if np.isnan(x).any() or np.isposinf(x).any() or np.isneginf(x).all():
+        return 0.0
+    m = x.max()
+    return float(math.exp(x[tok] - m) / np.exp(x - m).sum())
+
+
+def next_tokens(token: np.ndarray, state_out: np.ndarray, mask_token: int) -> np.ndarray:
+    """R10, the last line of Algorithm 1's step: positions in C_{t+1} and U_{t+1} take the
+    decoded token x^, positions in M_{t+1} keep the mask token."""
+    return np.where(np.asarray(state_out) == M, mask_token, np.asarray(token)).astype(np.int64)
+
+
 def next_state(c: float, tau_c: float, tau_u: float) -> int:
     """Eq. 8: c <= tau_c -> M; tau_c < c <= tau_u -> C; tau_u < c -> U."""
     if c <= tau_c:
@@ -286,11 +311,14 @@ class ScoreResult:
     promoted: list
     demoted: list
     counts: np.ndarray     # int64 [3]: M, C, U after the transition
+    p_cur: np.ndarray | None = None        # float64 [B] (R9), when cur_token is given
+    tokens_next: np.ndarray | None = None  # int64 [B] (R10), when mask_token is given
 
 
 def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray,
                 tau_c: float, tau_u: float, lam: float = LAMBDA_DEFAULT,
-                p0: float = P0_DEFAULT) -> ScoreResult:
+                p0: float = P0_DEFAULT, cur_token: np.ndarray | None = None,
+                mask_token: int | None = None) -> ScoreResult:
     """One block of Algorithm 1 after the forward pass (float64 except Eq. 7).
 
     logits_x / logits_s: [B, V] logits of x^i and s^i for every block position i.
@@ -298,6 +326,8 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
     2. C positions move by Eq. 8; those that reach U form P, those that reach M form D.
     3. M positions: w from P and D (Eq. 5, 6), mixed logits (Eq. 7), c and x^ from them.
     4. M and U positions move by Eq. 8.
+    Optional: p_cur of cur_token on each scored distribution (R9), and the next step's
+    tokens (R10) when mask_token is given.
     """
     B = len(state_in)
     st = np.where(state_in > 2, M, state_in).astype(np.int64)  # R7
@@ -306,6 +336,7 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
     valid = np.zeros(B, dtype=bool)
     new = np.zeros(B, dtype=np.int64)
     w_out = np.full(B, np.nan, dtype=np.float32)
+    p_cur = None if cur_token is None else np.zeros(B, dtype=np.float64)
 
     # 1-2: candidate and unmasked positions are verified from the shadow sequence.
     promoted, demoted = [], []
@@ -314,6 +345,8 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
             continue
         c, tok, ok = confidence(logits_s[i])
         conf[i], token[i], valid[i] = c, tok, ok
+        if p_cur is not None:
+            p_cur[i] = token_probability(logits_s[i], int(cur_token[i]))
         new[i] = next_state(c, tau_c, tau_u) if ok else M
         if st[i] == C:
             if new[i] == U:
@@ -331,11 +364,14 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
         mixed = mix_logits(logits_x[i], logits_s[i], w32)
         c, tok, ok = confidence(mixed)
         conf[i], token[i], valid[i] = c, tok, ok
+        if p_cur is not None:
+            p_cur[i] = token_probability(mixed, int(cur_token[i]))
         new[i] = next_state(c, tau_c, tau_u) if ok else M
 
     counts = np.array([(new == s).sum() for s in (M, C, U)], dtype=np.int64)
+    tokens_next = None if mask_token is None else next_tokens(token, new, mask_token)
     return ScoreResult(conf, token, new.astype(np.uint8), w_out, valid, promoted, demoted,
-                       counts)
+                       counts, p_cur, tokens_next)
 
 
 def top2_gap(row: np.ndarray) -> float:

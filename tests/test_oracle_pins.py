@@ -457,3 +457,66 @@ def test_score_block_fixed_weight_special_cases():
         assert res.w[r] == 1.0
         c, tok, _ = orc.confidence(lx[r])
         assert res.token[r] == tok and abs(res.conf[r] - c) < 1e-15
+
+
+# ---------------------------------------------------------------- R9, R10 (p_cur, tokens)
+def test_token_probability_closed_forms():
+    """A uniform row gives 1/V to every token; a planted row gives p to the peak and
+    (1 - p)/(V - 1) to the rest (float32 rounding of the log only)."""
+    V = 50
+    u = np.zeros(V, np.float32)
+    for tok in (0, 17, V - 1):
+        assert abs(orc.token_probability(u, tok) - 1.0 / V) < 1e-15
+    row = _peaked_row(V, 0.73, col=9)
+    assert abs(orc.token_probability(row, 9) - 0.73) < 1e-6
+    assert abs(orc.token_probability(row, 3) - 0.27 / (V - 1)) < 1e-7
+
+
+def test_token_probability_against_library_softmax():
+    rng = np.random.default_rng(5)
+    for V in (1, 2, 7, 300):
+        row = (rng.standard_normal(V) * 3).astype(np.float32)
+        ref = scipy.special.softmax(row.astype(np.float64))
+        got = np.array([orc.token_probability(row, t) for t in range(V)])
+        np.testing.assert_allclose(got, ref, rtol=1e-12, atol=0)
+        c, tok, _ = orc.confidence(row)
+        assert got[tok] == pytest.approx(c, rel=1e-12)   # Eq. 1: c = p(x^)
+
+
+def test_token_probability_out_of_range_and_invalid_rows():
+    row = np.zeros(8, np.float32)
+    assert orc.token_probability(row, -1) == 0.0 and orc.token_probability(row, 8) == 0.0
+    bad = row.copy()
+    bad[2] = np.nan
+    assert orc.token_probability(bad, 0) == 0.0
+    assert orc.token_probability(np.full(8, -np.inf, np.float32), 0) == 0.0
+
+
+def test_score_block_p_cur_uses_the_scored_distribution():
+    """C/U rows: p_cur on the shadow logits; M rows: on the mixed logits (with no C rows,
+    w = 1 and the mixture is the original logits)."""
+    rng = np.random.default_rng(12)
+    V = 96
+    state = np.array([M, U, M, U], dtype=np.uint8)
+    lx = ((rng.standard_normal((4, V)) * 2).astype(np.float32).view(np.uint32)
+          & np.uint32(0xFFFF0000)).view(np.float32)
+    ls = ((rng.standard_normal((4, V)) * 2).astype(np.float32).view(np.uint32)
+          & np.uint32(0xFFFF0000)).view(np.float32)
+    cur = np.array([3, 40, V, 0], np.int32)
+    res = orc.score_block(lx, ls, state, 0.4, 0.9, cur_token=cur)
+    assert res.p_cur[0] == pytest.approx(scipy.special.softmax(lx[0].astype(np.float64))[3], rel=1e-12)
+    assert res.p_cur[1] == pytest.approx(scipy.special.softmax(ls[1].astype(np.float64))[40], rel=1e-12)
+    assert res.p_cur[2] == 0.0                                   # token outside the vocabulary
+    assert res.p_cur[3] == pytest.approx(scipy.special.softmax(ls[3].astype(np.float64))[0], rel=1e-12)
+
+
+def test_next_tokens_fill_and_mask():
+    """The last line of Algorithm 1's step: C and U positions take x^, M positions the mask."""
+    tok = np.array([5, 7, 9, -1])
+    st = np.array([M, C, U, M], np.uint8)
+    assert list(orc.next_tokens(tok, st, 126336)) == [126336, 7, 9, 126336]
+    V = 32
+    rows = np.stack([_peaked_row(V, p, col=c) for p, c in ((0.95, 4), (0.6, 8), (0.1, 12))])
+    res = orc.score_block(rows, rows, np.array([U, C, U], np.uint8), 0.5, 0.8, mask_token=-7)
+    assert list(res.state_out) == [U, C, M]
+    assert list(res.tokens_next) == [4, 8, -7]
