@@ -166,7 +166,21 @@ typedef struct {
                                 No initial contents are needed. Calls that overlap on the
                                 GPU need separate workspaces.                              */
   size_t workspace_bytes;
+  /* Optional, the end of a step (each may be NULL):                                       */
+  const int32_t* cur_token;  /* device [rows] the token currently at each block position   */
+  float* p_cur;              /* device [rows] out: the probability the scored distribution
+                                (shadow logits for C/U rows, mixed logits for M rows) gives
+                                to cur_token; 0 for a token outside [0, vocab) or an invalid
+                                row. Needs cur_token.                                      */
+  int32_t* tokens;           /* device [rows] out: the next step's tokens, as the last line
+                                of Algorithm 1's step fills them: x^ where the new state is
+                                C or U, mask_token where it is M                           */
+  int32_t mask_token;        /* the mask token id written by `tokens`                      */
 } dard_score_args;
+
+/* In place: state_out may be the state_in buffer (the next step's states replace this
+ * step's), and conf can serve directly as the next step's prev_conf of dard_step_attention;
+ * tokens may be the buffer cur_token points to. */
 
 /* Bytes of workspace a call with these sizes needs (0 on invalid sizes). */
 size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs);

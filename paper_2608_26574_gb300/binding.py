@@ -45,7 +45,9 @@ class ScoreArgs(ctypes.Structure):
                 ("conf", ctypes.c_void_p), ("token", ctypes.c_void_p),
                 ("state_out", ctypes.c_void_p), ("w_out", ctypes.c_void_p),
                 ("counts", ctypes.c_void_p), ("status", ctypes.c_void_p),
-                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t)]
+                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+                ("cur_token", ctypes.c_void_p), ("p_cur", ctypes.c_void_p),
+                ("tokens", ctypes.c_void_p), ("mask_token", ctypes.c_int32)]
 
 
 class DardError(RuntimeError):
@@ -162,9 +164,11 @@ def dard_score_workspace_size(rows: int, vocab: int, num_seqs: int) -> int:
 
 def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, tau_u, lam, p0,
                               conf, token, state_out, workspace, w_out=None, counts=None,
-                              status=None, stream=None):
+                              status=None, stream=None, cur_token=None, p_cur=None,
+                              tokens=None, mask_token: int = 0):
     """Scoring and transition of every block row; logits [rows, V] with contiguous rows and
-    the same row pitch (``stride(0)``, at least V) in both tensors."""
+    the same row pitch (``stride(0)``, at least V) in both tensors. Optional end of step:
+    ``p_cur`` of ``cur_token``, and ``tokens`` (x^, or ``mask_token`` for rows ending in M)."""
     block_len = _host_i32(block_len)
     if logits_x.stride(0) != logits_s.stride(0) or logits_x.shape != logits_s.shape:
         raise ValueError("logits_x and logits_s need the same shape and row pitch")
@@ -181,6 +185,8 @@ def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, ta
     a.w_out, a.counts, a.status = _ptr(w_out), _ptr(counts), _ptr(status)
     a.workspace = _ptr(workspace)
     a.workspace_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    a.cur_token, a.p_cur, a.tokens = _ptr(cur_token), _ptr(p_cur), _ptr(tokens)
+    a.mask_token = mask_token
     _check(lib().dard_score_and_transition(ctypes.byref(a), _stream(stream)),
            "dard_score_and_transition")
 

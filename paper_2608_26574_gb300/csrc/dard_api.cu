@@ -181,6 +181,7 @@ dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
   if (rows > 0 && (!a->logits_x || !a->logits_s || !a->state_in || !a->conf || !a->token ||
                    !a->state_out))
     return fail(DARD_ERR_NULL, "a logits, state or output pointer is NULL");
+  if (a->p_cur && !a->cur_token) return fail(DARD_ERR_NULL, "p_cur needs cur_token");
   const int esz = a->dtype == DARD_BF16 ? 2 : 4;
   if (rows > 0 && (!aligned16(a->logits_x) || !aligned16(a->logits_s) ||
                    (a->row_stride * esz) % 16 != 0))
@@ -199,6 +200,11 @@ dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
   p.w_out = a->w_out;
   p.counts = a->counts;
   p.status = a->status;
+  p.cur_token = a->cur_token;
+  p.p_cur = a->p_cur;
+  p.tokens = a->tokens;
+  p.mask_token = a->mask_token;
+  p.state_in_place = static_cast<const void*>(a->state_out) == static_cast<const void*>(a->state_in);
   p.row_stride = a->row_stride;
   p.vocab = a->vocab;
   p.rows = static_cast<int32_t>(rows);

@@ -60,9 +60,15 @@ struct ScoreParams {
   uint8_t* state_out;
   float* w_out;
   int32_t* counts;
+  const int32_t* cur_token;  // optional: p_cur of this token
+  float* p_cur;              // optional
+  int32_t* tokens;           // optional: next step's tokens (x^, or mask_token for M)
+  int32_t mask_token;
+  int32_t state_in_place;    // state_out is the state_in buffer
   uint32_t* status;
   // workspace
-  uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 0 otherwise
+  uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 3 = an M row
+                       // (scored in pass 2), 0 otherwise
   int64_t row_stride;
   int32_t vocab, rows, num_seqs, nsplit, chunk;
   float tau_c, tau_u, lambda, p0;

@@ -236,9 +236,21 @@ __device__ __forceinline__ Acc merge_slots(const float4* slots, int nsplit) {
   return warp_merge(a);
 }
 
-// Eq. 1 and Eq. 8 on a merged row; writes conf / token / state and returns the new state.
+// The scored logit of the current token (p_cur), or NaN without one. lf(col) returns the
+// row's scored logit at col (shadow, or mixed for M rows).
+template <class LogitFn>
+__device__ __forceinline__ float current_logit(const ScoreParams& p, int row, LogitFn lf) {
+  if (p.p_cur == nullptr) return __int_as_float(0x7fc00000);
+  const int ct = p.cur_token[row];
+  return (ct >= 0 && ct < p.vocab) ? lf(ct) : -INFINITY;
+}
+
+// Eq. 1 and Eq. 8 on a merged row; writes conf / token / state, the optional p_cur (of the
+// current token's scored logit lc) and next-step token (x^, or the mask token for a row
+// that ends in M: the last line of Algorithm 1's step); returns the new state.
+template <bool kExtra>
 __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const Acc& a,
-                                            float w) {
+                                            float w, float lc) {
   const float z = a.s;
   const bool valid = isfinite(z) && z > 0.f;
   const float c = valid ? 1.0f / z : 0.f;
@@ -247,6 +259,11 @@ __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const
   p.token[row] = valid ? a.idx : -1;
   p.state_out[row] = static_cast<uint8_t>(ns);
   if (p.w_out) p.w_out[row] = w;
+  if (kExtra && p.p_cur) {
+    const float mL = a.m * kLog2e;
+    p.p_cur[row] = (valid && lc != -INFINITY) ? ex2_approx(fmaf(lc, kLog2e, -mL)) / z : 0.f;
+  }
+  if (kExtra && p.tokens) p.tokens[row] = ns == kStateM ? p.mask_token : a.idx;
   if (!valid && p.status) atomicOr(p.status, DARD_STATUS_INVALID_ROW);
   return ns;
 }
@@ -261,7 +278,8 @@ __device__ __forceinline__ void add_count(const ScoreParams& p, int seq, int sta
   if (p.counts != nullptr) atomicAdd(&p.counts[seq * 3 + state], 1);
 }
 
-template <class T, int VPT>
+// kExtra: the call asks for p_cur, next-step tokens or an in-place state update.
+template <class T, int VPT, bool kExtra>
 __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_constant__ ScoreParams p) {
   grid_dep_launch();  // pass 2 may start loading its logits right away
   __shared__ Acc s_acc[kWarps];
@@ -270,7 +288,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   const int row = blockIdx.y, split = blockIdx.x;  // split = rank in the row's cluster
   const int st = load_state(p, row, split == 0);
   if (st == kStateM) {  // uniform over the cluster: no CTA of it reaches the barrier
-    if (split == 0) p.pd_flag[row] = 0;
+    if (split == 0) p.pd_flag[row] = 3;  // pass 2's row (even if state_out overwrites it)
     return;
   }
   const char* rowp = static_cast<const char*>(p.ls) + static_cast<size_t>(row) * p.row_stride * T::kBytes;
@@ -289,16 +307,20 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   if (split != 0 || threadIdx.x >= 32) return;
   const Acc a = merge_slots(s_slots, p.nsplit);
   if (threadIdx.x == 0) {
-    const int ns = finalize_row(p, row, a, __int_as_float(0x7fc00000));
+    const float lc = !kExtra ? 0.f : current_logit(p, row, [&](int col) {
+      return T::scalar(rowp + static_cast<size_t>(col) * T::kBytes);
+    });
+    const int ns = finalize_row<kExtra>(p, row, a, __int_as_float(0x7fc00000), lc);
     p.pd_flag[row] = (st == kStateC) ? (ns == kStateU ? 1 : (ns == kStateM ? 2 : 0)) : 0;
   }
 }
 
-template <class T, int VPT>
+template <class T, int VPT, bool kExtra>
 __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_constant__ ScoreParams p) {
   __shared__ Acc s_acc[kWarps];
   __shared__ float4 s_slots[kScoreMaxSplit];
   __shared__ float s_w;
+  __shared__ bool s_m_row;
   const int row = blockIdx.y, split = blockIdx.x;
   const int st = load_state(p, row, false);
   const int seq = seq_of_row(p, row);
@@ -327,9 +349,13 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
 
   // Eq. 5-6: w from the verification outcomes of this block, computed by warp 0: each lane
   // sums lambda^|i-j| = 2^(|i-j| log2 lambda) over its positions, then a shuffle tree.
+  // With state_out aliasing state_in, a C or U row that pass 1 moved to M reads as M above;
+  // its own outcome byte (3 = an M row), loaded beside the others, tells them apart (only
+  // then: without aliasing the state read above is this step's).
   const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
   const int i = row - b0;
   if (threadIdx.x < 32) {
+    const int own = (kExtra && threadIdx.x == 0 && p.state_in_place) ? __ldcg(p.pd_flag + row) : 3;
     float pp = 0.f, dd = 0.f;
     for (int j = threadIdx.x; j < blen; j += 32) {
       const int f = __ldcg(p.pd_flag + b0 + j);
@@ -342,9 +368,17 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
       pp += __shfl_xor_sync(0xffffffffu, pp, off);
       dd += __shfl_xor_sync(0xffffffffu, dd, off);
     }
-    if (threadIdx.x == 0) s_w = __fdiv_rn(pp + p.p0, pp + dd + p.p0);
+    if (threadIdx.x == 0) {
+      s_w = __fdiv_rn(pp + p.p0, pp + dd + p.p0);
+      if (kExtra) s_m_row = own == 3;
+    }
   }
   __syncthreads();
+  if (kExtra && !s_m_row) {  // uniform over the cluster
+    if (split == 0 && p.counts != nullptr && threadIdx.x == 0)
+      add_count(p, seq, __ldcg(p.state_out + row));
+    return;
+  }
   const float w = s_w;
 
   // Eq. 7 in fp32, one rounding per operation: mix = ls + w * (lx - ls).
@@ -367,7 +401,14 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   cluster_publish(acc, split, s_slots);
   if (split != 0 || threadIdx.x >= 32) return;
   const Acc a = merge_slots(s_slots, p.nsplit);
-  if (threadIdx.x == 0) add_count(p, seq, finalize_row(p, row, a, w));
+  if (threadIdx.x == 0) {
+    const float lc = !kExtra ? 0.f : current_logit(p, row, [&](int col) {
+      const size_t off = static_cast<size_t>(col) * T::kBytes;
+      const float lx = T::scalar(xp + off), ls = T::scalar(sp + off);
+      return __fadd_rn(ls, __fmul_rn(w, __fsub_rn(lx, ls)));
+    });
+    add_count(p, seq, finalize_row<kExtra>(p, row, a, w, lc));
+  }
 }
 
 // Zeroes the counts when there are no rows at all (no pass runs).
@@ -387,11 +428,11 @@ cudaError_t allow_wide_clusters(F* kernel, std::atomic<uint64_t>& done) {
   return e;
 }
 
-template <class T, int VPT>
+template <class T, int VPT, bool kExtra>
 cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
   static std::atomic<uint64_t> done1{0}, done2{0};
-  cudaError_t e = allow_wide_clusters(score_pass1<T, VPT>, done1);
-  if (e == cudaSuccess) e = allow_wide_clusters(score_pass2<T, VPT>, done2);
+  cudaError_t e = allow_wide_clusters(score_pass1<T, VPT, kExtra>, done1);
+  if (e == cudaSuccess) e = allow_wide_clusters(score_pass2<T, VPT, kExtra>, done2);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.nsplit, p.rows);
@@ -407,10 +448,10 @@ cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, score_pass1<T, VPT>, p);
+  e = cudaLaunchKernelEx(&cfg, score_pass1<T, VPT, kExtra>, p);
   if (e != cudaSuccess) return e;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, score_pass2<T, VPT>, p);
+  return cudaLaunchKernelEx(&cfg, score_pass2<T, VPT, kExtra>, p);
 }
 
 }  // namespace
@@ -470,7 +511,9 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
     e = cudaGetLastError();
   }
   if (e == cudaSuccess && p.rows > 0) {
-    e = bf16 ? launch_pair<Bf16, 4>(p, stream) : launch_pair<F32, 4>(p, stream);
+    const bool extra = p.p_cur != nullptr || p.tokens != nullptr || p.state_in_place;
+    if (extra) e = bf16 ? launch_pair<Bf16, 4, true>(p, stream) : launch_pair<F32, 4, true>(p, stream);
+    else e = bf16 ? launch_pair<Bf16, 4, false>(p, stream) : launch_pair<F32, 4, false>(p, stream);
   }
   if (e != cudaSuccess) {
     snprintf(err, err_len, "scoring launch failed: %s", cudaGetErrorString(e));

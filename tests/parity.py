@@ -68,26 +68,33 @@ def compare_attention(wl, layer, o_host, sample=None, scale=None, rng=None):
     return float(e.max()), float(e.mean()), n
 
 
-def oracle_scores(wl):
+def oracle_scores(wl, cur_token=None, mask_token=None):
     """Per-sequence oracle results with the kernels' float32 parameters."""
     offs = wl.block_offsets()
     out = []
     for si, s in enumerate(wl.seqs):
         a, b = offs[si], offs[si + 1]
         out.append(orc.score_block(wl.logits_x[a:b], wl.logits_s[a:b], s.state,
-                                   f32(wl.tau_c), f32(wl.tau_u), f32(wl.lam), f32(wl.p0)))
+                                   f32(wl.tau_c), f32(wl.tau_u), f32(wl.lam), f32(wl.p0),
+                                   cur_token=None if cur_token is None else cur_token[a:b],
+                                   mask_token=mask_token))
     return out
 
 
-def compare_scores(wl, conf, token, state_out, w_out=None, counts=None):
+def compare_scores(wl, conf, token, state_out, w_out=None, counts=None, cur_token=None,
+                   p_cur=None, tokens_next=None, mask_token=None):
     """Checks the kernel outputs against the oracle. Exact: states and tokens, except rows
     whose oracle confidence lies within BORDER of a threshold (and, for a C row, the M rows
     of its block, whose w depends on it) and tokens of rows whose scored logits have a top-2
-    gap under NEAR_TIE. Returns a report dict; raises AssertionError on any mismatch."""
+    gap under NEAR_TIE. Optional: p_cur of cur_token (within CONF_TOL) and the next step's
+    tokens (exact, with the same exclusions as states and tokens). Returns a report dict;
+    raises AssertionError on any mismatch."""
     offs = wl.block_offsets()
     taus = (f32(wl.tau_c), f32(wl.tau_u))
     rep = {"rows": 0, "borderline": 0, "near_tie": 0, "max_conf_err": 0.0, "max_w_rel": 0.0}
-    for si, (s, res) in enumerate(zip(wl.seqs, oracle_scores(wl))):
+    results = oracle_scores(wl, cur_token=cur_token,
+                            mask_token=mask_token if tokens_next is not None else None)
+    for si, (s, res) in enumerate(zip(wl.seqs, results)):
         a, b = offs[si], offs[si + 1]
         st = np.where(s.state > 2, 0, s.state)
         border = np.array([min(abs(c - taus[0]), abs(c - taus[1])) < BORDER for c in res.conf],
@@ -118,6 +125,12 @@ def compare_scores(wl, conf, token, state_out, w_out=None, counts=None):
                 rep["near_tie"] += 1
             else:
                 assert token[r] == res.token[i], (si, i, token[r], res.token[i])
+                if tokens_next is not None:
+                    assert tokens_next[r] == res.tokens_next[i], (si, i, tokens_next[r])
+            if p_cur is not None:
+                perr = abs(float(p_cur[r]) - res.p_cur[i])
+                rep["max_p_cur_err"] = max(rep.get("max_p_cur_err", 0.0), perr)
+                assert perr <= CONF_TOL, (si, i, p_cur[r], res.p_cur[i])
             err = abs(float(conf[r]) - res.conf[i])
             rep["max_conf_err"] = max(rep["max_conf_err"], err)
             assert err <= CONF_TOL, (si, i, conf[r], res.conf[i])

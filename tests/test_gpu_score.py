@@ -3,6 +3,7 @@ import numpy as np
 import pytest
 import torch
 
+from paper_2608_26574_gb300 import binding as B
 from paper_2608_26574_gb300 import workloads as W
 from paper_2608_26574_gb300.device import DeviceStep
 
@@ -105,3 +106,48 @@ def test_score_threshold_edges():
     for tau in ((0.6, 0.6), (0.0, 1.0), (0.0, 0.0), (1.0, 1.0)):
         wl = W.custom(specs, 1, 1, 64, vocab=2000, seed=11, tau=tau, logit_std=1.0)
         _check(wl, _run(wl)[1])
+
+
+def _end_of_step(ds, cur, mask_token, in_place):
+    """Scores with p_cur of `cur` and next-step tokens; with in_place, state_out is the
+    state_in buffer and tokens overwrite the cur_token buffer."""
+    wl = ds.wl
+    rows = ds.state.numel()
+    p_cur = torch.full((rows,), -1.0, dtype=torch.float32, device=ds.state.device)
+    if in_place:
+        state_io = ds.state.clone()
+        tokens = cur.clone()
+        cur_in, st_out = tokens, state_io
+    else:
+        state_io, tokens, cur_in, st_out = ds.state, torch.empty_like(cur), cur, ds.state_out
+    B.dard_score_and_transition(ds.lx, ds.ls, ds.block_len, state_io, wl.tau_c, wl.tau_u, wl.lam,
+                                wl.p0, ds.conf, ds.token, st_out, ds.workspace, w_out=ds.w_out,
+                                counts=ds.counts, status=ds.status, cur_token=cur_in,
+                                p_cur=p_cur, tokens=tokens, mask_token=mask_token)
+    torch.cuda.synchronize()
+    return (p_cur.cpu().numpy(), tokens.cpu().numpy(), st_out.cpu().numpy())
+
+
+@pytest.mark.parametrize("name", ["tiny", "8b", "gqa", "mm", "ragged"])
+@pytest.mark.parametrize("in_place", [False, True])
+def test_score_end_of_step(name, in_place):
+    """p_cur of the current token on each row's scored distribution, the next step's tokens
+    (x^, or the mask token for rows ending in M), with the state updated in place or not."""
+    wl = W.make(name, logits="spanning", attention=False)
+    ds = DeviceStep(wl, attention=False)
+    rng = np.random.default_rng(31)
+    rows = wl.total_block
+    cur = rng.integers(-2, wl.vocab + 2, size=rows).astype(np.int32)
+    # a third of the rows hold their current argmax, so that p_cur = c is exercised too
+    for si, res in enumerate(P.oracle_scores(wl)):
+        a = wl.block_offsets()[si]
+        for i in range(0, len(res.token), 3):
+            cur[a + i] = res.token[i]
+    cur_d = torch.from_numpy(cur).to(ds.state.device)
+    mask_token = 126336
+    p_cur, tokens, st = _end_of_step(ds, cur_d, mask_token, in_place)
+    conf, token, w, counts = (t.cpu().numpy() for t in (ds.conf, ds.token, ds.w_out, ds.counts))
+    rep = P.compare_scores(wl, conf, token, st, w_out=w, counts=counts, cur_token=cur,
+                           p_cur=p_cur, tokens_next=tokens, mask_token=mask_token)
+    assert int(ds.status.item()) == 0
+    print(name, in_place, rep)
