@@ -36,7 +36,14 @@ Readings of points the paper leaves open (each is listed in the design doc):
       for C and U positions, mixed logits for M positions) gives to the token currently at
       the position; 0 for a token outside the vocabulary or an invalid row;
   R10 the token update that closes a step of Algorithm 1: positions that end the step in
-      M hold the mask token again, every other position holds its new prediction x^.
+      M hold the mask token again, every other position holds its new prediction x^;
+  R11 the ordering variants of the attention-mask ablation of Sec. 5 (bidirectional, l2r,
+      entropy, margin) differ only in the key that Eq. 3 compares: bidirectional = equal
+      keys (every C pair attends both ways), l2r = minus the block position (earlier
+      positions rank higher), entropy = minus the entropy of the scored distribution (in
+      nats; more certain ranks higher), margin = p(x^) minus the second-largest probability
+      (a repeated maximum gives 0; a one-entry vocabulary gives 1). An invalid row (R6) has
+      entropy 0 and margin 0.
 
 Parity pins: every function here is pinned by ``tests/test_oracle_pins.py`` except where
 a docstring says "parity unpinned".
@@ -259,6 +266,40 @@ def token_probability(logits_row: np.ndarray, tok: int) -> float:
     return float(math.exp(x[tok] - m) / np.exp(x - m).sum())
 
 
+def entropy(logits_row: np.ndarray) -> float:
+    """R11: -sum_v p_v ln p_v of the softmax of the row (float64); 0 for an invalid row."""
+    x = logits_row.astype(np.float64)
+    if np.isnan(x).any() or np.isposinf(x).any() or np.isneginf(x).all():
+        return 0.0
+    p = np.exp(x - x.max())
+    p /= p.sum()
+    nz = p > 0
+    return float(-(p[nz] * np.log(p[nz])).sum())
+
+
+def margin(logits_row: np.ndarray) -> float:
+    """R11: p(x^) minus the second-largest probability (float64); 0 for an invalid row."""
+    x = logits_row.astype(np.float64)
+    if np.isnan(x).any() or np.isposinf(x).any() or np.isneginf(x).all():
+        return 0.0
+    p = np.exp(x - x.max())
+    p /= p.sum()
+    if len(p) < 2:
+        return float(p[0])
+    top = np.sort(p)
+    return float(top[-1] - top[-2])
+
+
+# Ordering modes of R11 (the key Eq. 3 compares in the next step)
+ORDER_CONFIDENCE, ORDER_BIDIR, ORDER_L2R, ORDER_ENTROPY, ORDER_MARGIN = 0, 1, 2, 3, 4
+
+
+def order_key(mode: int, c: float, h: float, mg: float, i: int) -> float:
+    """R11: the next step's ordering key of block position i."""
+    return {ORDER_CONFIDENCE: c, ORDER_BIDIR: 0.0, ORDER_L2R: -float(i),
+            ORDER_ENTROPY: -h, ORDER_MARGIN: mg}[mode]
+
+
 def next_tokens(token: np.ndarray, state_out: np.ndarray, mask_token: int) -> np.ndarray:
     """R10, the last line of Algorithm 1's step: positions in C_{t+1} and U_{t+1} take the
     decoded token x^, positions in M_{t+1} keep the mask token."""
@@ -313,6 +354,8 @@ class ScoreResult:
     counts: np.ndarray     # int64 [3]: M, C, U after the transition
     p_cur: np.ndarray | None = None        # float64 [B] (R9), when cur_token is given
     tokens_next: np.ndarray | None = None  # int64 [B] (R10), when mask_token is given
+    entropy: np.ndarray | None = None      # float64 [B] (R11) of each scored distribution
+    margin: np.ndarray | None = None       # float64 [B] (R11)
 
 
 def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray,
@@ -332,6 +375,8 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
     B = len(state_in)
     st = np.where(state_in > 2, M, state_in).astype(np.int64)  # R7
     conf = np.zeros(B, dtype=np.float64)
+    ent = np.zeros(B, dtype=np.float64)
+    mgn = np.zeros(B, dtype=np.float64)
     token = np.full(B, -1, dtype=np.int64)
     valid = np.zeros(B, dtype=bool)
     new = np.zeros(B, dtype=np.int64)
@@ -345,6 +390,7 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
             continue
         c, tok, ok = confidence(logits_s[i])
         conf[i], token[i], valid[i] = c, tok, ok
+        ent[i], mgn[i] = entropy(logits_s[i]), margin(logits_s[i])
         if p_cur is not None:
             p_cur[i] = token_probability(logits_s[i], int(cur_token[i]))
         new[i] = next_state(c, tau_c, tau_u) if ok else M
@@ -364,6 +410,7 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
         mixed = mix_logits(logits_x[i], logits_s[i], w32)
         c, tok, ok = confidence(mixed)
         conf[i], token[i], valid[i] = c, tok, ok
+        ent[i], mgn[i] = entropy(mixed), margin(mixed)
         if p_cur is not None:
             p_cur[i] = token_probability(mixed, int(cur_token[i]))
         new[i] = next_state(c, tau_c, tau_u) if ok else M
@@ -371,7 +418,7 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
     counts = np.array([(new == s).sum() for s in (M, C, U)], dtype=np.int64)
     tokens_next = None if mask_token is None else next_tokens(token, new, mask_token)
     return ScoreResult(conf, token, new.astype(np.uint8), w_out, valid, promoted, demoted,
-                       counts, p_cur, tokens_next)
+                       counts, p_cur, tokens_next, ent, mgn)
 
 
 def top2_gap(row: np.ndarray) -> float:

@@ -13,6 +13,7 @@ import os
 import numpy as np
 import pytest
 import scipy.special
+import scipy.stats
 import torch
 
 import oracle as orc
@@ -520,3 +521,50 @@ def test_next_tokens_fill_and_mask():
     res = orc.score_block(rows, rows, np.array([U, C, U], np.uint8), 0.5, 0.8, mask_token=-7)
     assert list(res.state_out) == [U, C, M]
     assert list(res.tokens_next) == [4, 8, -7]
+
+
+# ---------------------------------------------------------------- R11 (ordering variants)
+def test_entropy_and_margin_closed_forms():
+    V = 40
+    u = np.zeros(V, np.float32)
+    assert orc.entropy(u) == pytest.approx(math.log(V), rel=1e-12)
+    assert orc.margin(u) == 0.0
+    p = 0.7
+    row = _peaked_row(V, p, col=5)
+    q = (1 - p) / (V - 1)
+    assert orc.entropy(row) == pytest.approx(-p * math.log(p) - (1 - p) * math.log(q), rel=1e-6)
+    assert orc.margin(row) == pytest.approx(p - q, rel=1e-6)
+    two = np.zeros(V, np.float32)
+    two[[3, 9]] = 4.0                               # a repeated maximum: margin 0
+    assert orc.margin(two) == 0.0
+    assert orc.entropy(np.zeros(1, np.float32)) == 0.0 and orc.margin(np.zeros(1, np.float32)) == 1.0
+    bad = u.copy()
+    bad[0] = np.nan
+    assert orc.entropy(bad) == 0.0 and orc.margin(bad) == 0.0
+
+
+def test_entropy_and_margin_against_library():
+    rng = np.random.default_rng(8)
+    for V in (2, 17, 500):
+        row = (rng.standard_normal(V) * 2.5).astype(np.float32)
+        p = scipy.special.softmax(row.astype(np.float64))
+        assert orc.entropy(row) == pytest.approx(float(scipy.stats.entropy(p)), rel=1e-10)
+        srt = np.sort(p)
+        assert orc.margin(row) == pytest.approx(srt[-1] - srt[-2], rel=1e-10)
+
+
+def test_order_keys_reproduce_the_ablation_orderings():
+    """Eq. 3 with the R11 keys: equal keys make every C pair mutual (bidirectional); minus
+    the position gives left-to-right causal order among C positions."""
+    B = 6
+    st = np.full(B, C, np.uint8)
+    for mode, want in ((orc.ORDER_BIDIR, lambda i, j: True), (orc.ORDER_L2R, lambda i, j: j <= i)):
+        keys = np.array([orc.order_key(mode, 0.5, 1.0, 0.2, i) for i in range(B)], np.float32)
+        for i in range(B):
+            sees_shadow = orc.sees_shadow_copy("x", i, st, keys)
+            for j in range(B):
+                if j != i:
+                    assert (not sees_shadow[j]) == want(i, j), (mode, i, j)
+    assert orc.order_key(orc.ORDER_CONFIDENCE, 0.7, 2.0, 0.1, 3) == 0.7
+    assert orc.order_key(orc.ORDER_ENTROPY, 0.7, 2.0, 0.1, 3) == -2.0
+    assert orc.order_key(orc.ORDER_MARGIN, 0.7, 2.0, 0.1, 3) == 0.1
