@@ -58,6 +58,21 @@ typedef enum {
 
 typedef enum { DARD_F32 = 0, DARD_BF16 = 1 } dard_dtype;
 
+/* Orderings of candidate tokens in the mask (Eq. 3 compares one key per block position).
+ * The attention-mask ablation of Sec. 5 compares DARD's confidence ordering with a
+ * bidirectional mask and with left-to-right, entropy and margin orderings; each is a choice
+ * of key, which the scoring call can write for the next step (dard_score_args.order_key):
+ *   CONFIDENCE  c_t (the paper's DARD)          BIDIR   0 (equal keys: every C pair attends
+ *   L2R         minus the block position          both ways, Eq. 3 ties being mutual)
+ *   ENTROPY     minus the entropy (nats)        MARGIN  p(x^) minus the second probability */
+typedef enum {
+  DARD_ORDER_CONFIDENCE = 0,
+  DARD_ORDER_BIDIR = 1,
+  DARD_ORDER_L2R = 2,
+  DARD_ORDER_ENTROPY = 3,
+  DARD_ORDER_MARGIN = 4
+} dard_order_mode;
+
 /* Bits of the optional device status word (OR-ed in, never cleared by the library). */
 #define DARD_STATUS_BAD_STATE 0x1u     /* a state byte > 2 (treated as M)                    */
 #define DARD_STATUS_BAD_SHADOW 0x2u    /* shadow_src outside its block or repeated (row
@@ -176,6 +191,13 @@ typedef struct {
                                 of Algorithm 1's step fills them: x^ where the new state is
                                 C or U, mask_token where it is M                           */
   int32_t mask_token;        /* the mask token id written by `tokens`                      */
+  float* entropy;            /* device [rows] out: entropy (nats) of the scored
+                                distribution; 0 for an invalid row                         */
+  float* margin;             /* device [rows] out: p(x^) minus the second-largest
+                                probability (a repeated maximum gives 0); 0 if invalid     */
+  float* order_key;          /* device [rows] out: the next step's ordering key, to pass as
+                                dard_attn_args.prev_conf, per order_mode                   */
+  int32_t order_mode;        /* dard_order_mode of order_key                               */
 } dard_score_args;
 
 /* In place: state_out may be the state_in buffer (the next step's states replace this

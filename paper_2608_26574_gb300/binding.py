@@ -17,6 +17,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libdard.so")
 
 DARD_F32, DARD_BF16 = 0, 1
+ORDER_CONFIDENCE, ORDER_BIDIR, ORDER_L2R, ORDER_ENTROPY, ORDER_MARGIN = 0, 1, 2, 3, 4
 STATUS_BAD_STATE, STATUS_BAD_SHADOW, STATUS_INVALID_ROW, STATUS_TIMEOUT = 0x1, 0x2, 0x4, 0x8
 MAX_SEQS, MAX_BLOCK = 256, 128
 SCORE_NOALLOC_MAX_ROWS = 8192
@@ -47,7 +48,9 @@ class ScoreArgs(ctypes.Structure):
                 ("counts", ctypes.c_void_p), ("status", ctypes.c_void_p),
                 ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
                 ("cur_token", ctypes.c_void_p), ("p_cur", ctypes.c_void_p),
-                ("tokens", ctypes.c_void_p), ("mask_token", ctypes.c_int32)]
+                ("tokens", ctypes.c_void_p), ("mask_token", ctypes.c_int32),
+                ("entropy", ctypes.c_void_p), ("margin", ctypes.c_void_p),
+                ("order_key", ctypes.c_void_p), ("order_mode", ctypes.c_int32)]
 
 
 class DardError(RuntimeError):
@@ -165,10 +168,12 @@ def dard_score_workspace_size(rows: int, vocab: int, num_seqs: int) -> int:
 def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, tau_u, lam, p0,
                               conf, token, state_out, workspace, w_out=None, counts=None,
                               status=None, stream=None, cur_token=None, p_cur=None,
-                              tokens=None, mask_token: int = 0):
+                              tokens=None, mask_token: int = 0, entropy=None, margin=None,
+                              order_key=None, order_mode: int = ORDER_CONFIDENCE):
     """Scoring and transition of every block row; logits [rows, V] with contiguous rows and
     the same row pitch (``stride(0)``, at least V) in both tensors. Optional end of step:
-    ``p_cur`` of ``cur_token``, and ``tokens`` (x^, or ``mask_token`` for rows ending in M)."""
+    ``p_cur`` of ``cur_token``, and ``tokens`` (x^, or ``mask_token`` for rows ending in M);
+    ``entropy``, ``margin`` and the next step's ``order_key`` for ``order_mode``."""
     block_len = _host_i32(block_len)
     if logits_x.stride(0) != logits_s.stride(0) or logits_x.shape != logits_s.shape:
         raise ValueError("logits_x and logits_s need the same shape and row pitch")
@@ -187,6 +192,8 @@ def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, ta
     a.workspace_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     a.cur_token, a.p_cur, a.tokens = _ptr(cur_token), _ptr(p_cur), _ptr(tokens)
     a.mask_token = mask_token
+    a.entropy, a.margin, a.order_key = _ptr(entropy), _ptr(margin), _ptr(order_key)
+    a.order_mode = order_mode
     _check(lib().dard_score_and_transition(ctypes.byref(a), _stream(stream)),
            "dard_score_and_transition")
 

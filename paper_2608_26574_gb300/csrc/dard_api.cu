@@ -182,6 +182,8 @@ dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
                    !a->state_out))
     return fail(DARD_ERR_NULL, "a logits, state or output pointer is NULL");
   if (a->p_cur && !a->cur_token) return fail(DARD_ERR_NULL, "p_cur needs cur_token");
+  if (a->order_mode < DARD_ORDER_CONFIDENCE || a->order_mode > DARD_ORDER_MARGIN)
+    return fail(DARD_ERR_VALUE, "order_mode %d is not a dard_order_mode", a->order_mode);
   const int esz = a->dtype == DARD_BF16 ? 2 : 4;
   if (rows > 0 && (!aligned16(a->logits_x) || !aligned16(a->logits_s) ||
                    (a->row_stride * esz) % 16 != 0))
@@ -205,6 +207,10 @@ dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
   p.tokens = a->tokens;
   p.mask_token = a->mask_token;
   p.state_in_place = static_cast<const void*>(a->state_out) == static_cast<const void*>(a->state_in);
+  p.entropy = a->entropy;
+  p.margin = a->margin;
+  p.order_key = a->order_key;
+  p.order_mode = a->order_mode;
   p.row_stride = a->row_stride;
   p.vocab = a->vocab;
   p.rows = static_cast<int32_t>(rows);

@@ -65,6 +65,10 @@ struct ScoreParams {
   int32_t* tokens;           // optional: next step's tokens (x^, or mask_token for M)
   int32_t mask_token;
   int32_t state_in_place;    // state_out is the state_in buffer
+  float* entropy;            // optional
+  float* margin;             // optional
+  float* order_key;          // optional: next step's key per order_mode
+  int32_t order_mode;
   uint32_t* status;
   // workspace
   uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 3 = an M row

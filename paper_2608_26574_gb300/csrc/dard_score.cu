@@ -17,6 +17,7 @@
 // dependent of pass 1: its CTAs load their logits while pass 1 finishes and only then
 // wait for pass 1's results.
 #include <atomic>
+#include <type_traits>
 #include <cfloat>
 #include <climits>
 #include <cmath>
@@ -216,6 +217,120 @@ __device__ __forceinline__ int load_state(const ScoreParams& p, int row, bool re
   return s;
 }
 
+// ---- the extended summary of the end-of-step variant: also the entropy sum
+// h = sum exp(x - m) (x - m) and the second-largest value m2 (a repeated maximum counts as
+// the second), for the entropy and the margin of the ordering variants.
+struct AccX {
+  float m;   // running maximum
+  float s;   // sum of exp(x - m)
+  int idx;   // lowest index attaining m
+  float h;   // sum of exp(x - m) * (x - m)
+  float m2;  // second-largest value
+};
+
+__device__ __forceinline__ AccX accx_init() { return {-INFINITY, 0.f, INT_MAX, 0.f, -INFINITY}; }
+
+// Re-expresses (s, h) of maximum m_old against the larger maximum m_new.
+__device__ __forceinline__ void accx_rescale(float& s, float& h, float m_old, float m_new) {
+  if (m_old == -INFINITY) {
+    s = 0.f;
+    h = 0.f;
+    return;
+  }
+  const float d = m_old - m_new;  // <= 0
+  const float f = ex2_approx(d * kLog2e);
+  h = f * fmaf(d, s, h);
+  s = s * f;
+}
+
+__device__ __forceinline__ AccX accx_merge(const AccX& a, const AccX& b) {
+  const bool b_wins = (b.m > a.m) || (b.m == a.m && b.idx < a.idx);
+  const AccX hi = b_wins ? b : a;
+  AccX lo = b_wins ? a : b;
+  accx_rescale(lo.s, lo.h, lo.m, hi.m);
+  return {hi.m, hi.s + lo.s, hi.idx, hi.h + lo.h, fmaxf(fmaxf(a.m2, b.m2), lo.m)};
+}
+
+__device__ __forceinline__ AccX warp_merge(AccX a) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    AccX b;
+    b.m = __shfl_xor_sync(0xffffffffu, a.m, off);
+    b.s = __shfl_xor_sync(0xffffffffu, a.s, off);
+    b.idx = __shfl_xor_sync(0xffffffffu, a.idx, off);
+    b.h = __shfl_xor_sync(0xffffffffu, a.h, off);
+    b.m2 = __shfl_xor_sync(0xffffffffu, a.m2, off);
+    a = accx_merge(a, b);
+  }
+  return a;
+}
+
+template <class T, int VPT, bool kTail, class ValFn>
+__device__ __forceinline__ void fold_round(AccX& acc, int base, int limit, ValFn val) {
+  auto get = [&](int v, int e) {
+    const float x = val(v, e);
+    if (!kTail) return x;
+    const int i = base + (v * kScoreThreads + static_cast<int>(threadIdx.x)) * T::W + e;
+    return i < limit ? x : -INFINITY;
+  };
+  float m = -INFINITY, m2 = -INFINITY;
+  int idx = INT_MAX;
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+#pragma unroll
+    for (int e = 0; e < T::W; ++e) {
+      const float x = get(v, e);
+      if (x > m) {
+        m2 = m;
+        m = x;
+        idx = base + (v * kScoreThreads + static_cast<int>(threadIdx.x)) * T::W + e;
+      } else {
+        m2 = fmaxf(m2, x);
+      }
+    }
+  }
+  const float m2_all = fmaxf(fmaxf(acc.m2, m2), fminf(acc.m, m));
+  if (m > acc.m) {
+    accx_rescale(acc.s, acc.h, acc.m, m);
+    acc.m = m;
+    acc.idx = idx;
+  }
+  acc.m2 = m2_all;
+  if (acc.m == -INFINITY) return;
+  const float mL = acc.m * kLog2e;
+  float s = 0.f, h = 0.f;
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+#pragma unroll
+    for (int e = 0; e < T::W; ++e) {
+      const float x = get(v, e);
+      const float ex = ex2_approx(fmaf(x, kLog2e, -mL));
+      s += ex;
+      h = fmaf(ex, fmaxf(x - acc.m, -1e30f), h);  // -inf elements add 0, not NaN
+    }
+  }
+  acc.s += s;
+  acc.h += h;
+}
+
+template <class T, int VPT, class ValFn>
+__device__ __forceinline__ void fold(AccX& acc, int base, int limit, ValFn val) {
+  if (base + kScoreThreads * VPT * T::W <= limit) fold_round<T, VPT, false>(acc, base, limit, val);
+  else fold_round<T, VPT, true>(acc, base, limit, val);
+}
+
+__device__ __forceinline__ AccX block_merge(AccX a, AccX* smem) {
+  a = warp_merge(a);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) smem[warp] = a;
+  __syncthreads();
+  if (warp == 0) {
+    a = lane < kWarps ? smem[lane] : accx_init();
+    a = warp_merge(a);
+  }
+  return a;  // valid in warp 0
+}
+
 // Sends this CTA's partial (warp 0 holds it) to slot `split` of the leader CTA (cluster
 // rank 0), then synchronises the cluster; afterwards the leader's slots are complete.
 __device__ __forceinline__ void cluster_publish(const Acc& a, int split, float4* slots) {
@@ -224,17 +339,39 @@ __device__ __forceinline__ void cluster_publish(const Acc& a, int split, float4*
                   0.f);
   cluster_sync();
 }
+// The extended summary uses the slot pair (split, kScoreMaxSplit + split).
+__device__ __forceinline__ void cluster_publish(const AccX& a, int split, float4* slots) {
+  if (threadIdx.x == 0) {
+    st_cluster_v4(map_shared_rank(smem_u32(&slots[split]), 0), a.m, a.s, __int_as_float(a.idx),
+                  a.h);
+    st_cluster_v4(map_shared_rank(smem_u32(&slots[kScoreMaxSplit + split]), 0), a.m2, 0.f, 0.f,
+                  0.f);
+  }
+  cluster_sync();
+}
 
 // Merges the leader's slots in split order (warp 0); returns the row summary in lane 0.
-__device__ __forceinline__ Acc merge_slots(const float4* slots, int nsplit) {
+__device__ __forceinline__ void merge_slots(const float4* slots, int nsplit, Acc& out) {
   Acc a{-INFINITY, 0.f, INT_MAX};
   const int lane = threadIdx.x & 31;
   if (lane < nsplit) {
     const float4 v = slots[lane];
     a = Acc{v.x, v.y, __float_as_int(v.z)};
   }
-  return warp_merge(a);
+  out = warp_merge(a);
 }
+__device__ __forceinline__ void merge_slots(const float4* slots, int nsplit, AccX& out) {
+  AccX a = accx_init();
+  const int lane = threadIdx.x & 31;
+  if (lane < nsplit) {
+    const float4 v = slots[lane], v2 = slots[kScoreMaxSplit + lane];
+    a = AccX{v.x, v.y, __float_as_int(v.z), v.w, v2.x};
+  }
+  out = warp_merge(a);
+}
+
+__device__ __forceinline__ Acc acc_init(Acc*) { return {-INFINITY, 0.f, INT_MAX}; }
+__device__ __forceinline__ AccX acc_init(AccX*) { return accx_init(); }
 
 // The scored logit of the current token (p_cur), or NaN without one. lf(col) returns the
 // row's scored logit at col (shadow, or mixed for M rows).
@@ -248,8 +385,8 @@ __device__ __forceinline__ float current_logit(const ScoreParams& p, int row, Lo
 // Eq. 1 and Eq. 8 on a merged row; writes conf / token / state, the optional p_cur (of the
 // current token's scored logit lc) and next-step token (x^, or the mask token for a row
 // that ends in M: the last line of Algorithm 1's step); returns the new state.
-template <bool kExtra>
-__device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const Acc& a,
+template <bool kExtra, class A>
+__device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const A& a,
                                             float w, float lc) {
   const float z = a.s;
   const bool valid = isfinite(z) && z > 0.f;
@@ -264,6 +401,20 @@ __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const
     p.p_cur[row] = (valid && lc != -INFINITY) ? ex2_approx(fmaf(lc, kLog2e, -mL)) / z : 0.f;
   }
   if (kExtra && p.tokens) p.tokens[row] = ns == kStateM ? p.mask_token : a.idx;
+  if constexpr (kExtra) {
+    // entropy (nats) and margin of the scored distribution, the next step's ordering key
+    const float hnat = valid ? logf(z) - a.h / z : 0.f;
+    const float mg = valid ? (1.0f - ex2_approx((a.m2 - a.m) * kLog2e)) / z : 0.f;
+    if (p.entropy) p.entropy[row] = hnat;
+    if (p.margin) p.margin[row] = mg;
+    if (p.order_key) {
+      const int i = row - p.blk_off[seq_of_row(p, row)];
+      p.order_key[row] = p.order_mode == DARD_ORDER_BIDIR ? 0.f
+                       : p.order_mode == DARD_ORDER_L2R ? -static_cast<float>(i)
+                       : p.order_mode == DARD_ORDER_ENTROPY ? -hnat
+                       : p.order_mode == DARD_ORDER_MARGIN ? mg : c;
+    }
+  }
   if (!valid && p.status) atomicOr(p.status, DARD_STATUS_INVALID_ROW);
   return ns;
 }
@@ -282,8 +433,9 @@ __device__ __forceinline__ void add_count(const ScoreParams& p, int seq, int sta
 template <class T, int VPT, bool kExtra>
 __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_constant__ ScoreParams p) {
   grid_dep_launch();  // pass 2 may start loading its logits right away
-  __shared__ Acc s_acc[kWarps];
-  __shared__ float4 s_slots[kScoreMaxSplit];
+  using A = std::conditional_t<kExtra, AccX, Acc>;
+  __shared__ A s_acc[kWarps];
+  __shared__ float4 s_slots[2 * kScoreMaxSplit];
   zero_counts(p);
   const int row = blockIdx.y, split = blockIdx.x;  // split = rank in the row's cluster
   const int st = load_state(p, row, split == 0);
@@ -294,7 +446,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   const char* rowp = static_cast<const char*>(p.ls) + static_cast<size_t>(row) * p.row_stride * T::kBytes;
   const int c0 = split * p.chunk;
   const int c1 = min(p.vocab, c0 + p.chunk);
-  Acc acc{-INFINITY, 0.f, INT_MAX};
+  A acc = acc_init(static_cast<A*>(nullptr));
   for (int base = c0; base < c1; base += kScoreThreads * VPT * T::W) {
     uint4 r[VPT];
 #pragma unroll
@@ -305,7 +457,8 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   acc = block_merge(acc, s_acc);
   cluster_publish(acc, split, s_slots);
   if (split != 0 || threadIdx.x >= 32) return;
-  const Acc a = merge_slots(s_slots, p.nsplit);
+  A a;
+  merge_slots(s_slots, p.nsplit, a);
   if (threadIdx.x == 0) {
     const float lc = !kExtra ? 0.f : current_logit(p, row, [&](int col) {
       return T::scalar(rowp + static_cast<size_t>(col) * T::kBytes);
@@ -317,8 +470,9 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
 
 template <class T, int VPT, bool kExtra>
 __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_constant__ ScoreParams p) {
-  __shared__ Acc s_acc[kWarps];
-  __shared__ float4 s_slots[kScoreMaxSplit];
+  using A = std::conditional_t<kExtra, AccX, Acc>;
+  __shared__ A s_acc[kWarps];
+  __shared__ float4 s_slots[2 * kScoreMaxSplit];
   __shared__ float s_w;
   __shared__ bool s_m_row;
   const int row = blockIdx.y, split = blockIdx.x;
@@ -386,7 +540,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
     const float lx = T::get(vx, e), ls = T::get(vs, e);
     return __fadd_rn(ls, __fmul_rn(w, __fsub_rn(lx, ls)));
   };
-  Acc acc{-INFINITY, 0.f, INT_MAX};
+  A acc = acc_init(static_cast<A*>(nullptr));
   fold<T, VPT>(acc, c0, c1, [&](int v, int e) { return mix(rx[v], rs[v], e); });
   for (int base = c0 + kScoreThreads * VPT * T::W; base < c1; base += kScoreThreads * VPT * T::W) {
 #pragma unroll
@@ -400,7 +554,8 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   acc = block_merge(acc, s_acc);
   cluster_publish(acc, split, s_slots);
   if (split != 0 || threadIdx.x >= 32) return;
-  const Acc a = merge_slots(s_slots, p.nsplit);
+  A a;
+  merge_slots(s_slots, p.nsplit, a);
   if (threadIdx.x == 0) {
     const float lc = !kExtra ? 0.f : current_logit(p, row, [&](int col) {
       const size_t off = static_cast<size_t>(col) * T::kBytes;
@@ -511,7 +666,8 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
     e = cudaGetLastError();
   }
   if (e == cudaSuccess && p.rows > 0) {
-    const bool extra = p.p_cur != nullptr || p.tokens != nullptr || p.state_in_place;
+    const bool extra = p.p_cur != nullptr || p.tokens != nullptr || p.state_in_place ||
+                       p.entropy != nullptr || p.margin != nullptr || p.order_key != nullptr;
     if (extra) e = bf16 ? launch_pair<Bf16, 4, true>(p, stream) : launch_pair<F32, 4, true>(p, stream);
     else e = bf16 ? launch_pair<Bf16, 4, false>(p, stream) : launch_pair<F32, 4, false>(p, stream);
   }

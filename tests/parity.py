@@ -9,6 +9,9 @@ BORDER = 1e-5      # |c - tau| below this: the transition may legitimately go ei
 NEAR_TIE = 1e-3    # top-2 logit gap below this: the argmax may legitimately differ
 CONF_TOL = 1e-4    # confidences, fp32 accumulation
 W_REL = 4e-6       # guidance weight: fp32 sum of at most 128 terms against fp64
+# entropy (nats): ln Z - h/Z from two fp32 sums over V terms (Z, h = sum e^(x-m)(x-m)); their
+# relative rounding stays near 1e-5 at V = 152064, and h/Z is at most ln V < 12
+ENTROPY_TOL = 1e-3
 ATT_MAX_ABS = 2e-2
 ATT_MEAN_ABS = 1e-2
 
@@ -82,7 +85,8 @@ def oracle_scores(wl, cur_token=None, mask_token=None):
 
 
 def compare_scores(wl, conf, token, state_out, w_out=None, counts=None, cur_token=None,
-                   p_cur=None, tokens_next=None, mask_token=None):
+                   p_cur=None, tokens_next=None, mask_token=None, entropy=None, margin=None,
+                   order_key=None, order_mode=0):
     """Checks the kernel outputs against the oracle. Exact: states and tokens, except rows
     whose oracle confidence lies within BORDER of a threshold (and, for a C row, the M rows
     of its block, whose w depends on it) and tokens of rows whose scored logits have a top-2
@@ -127,6 +131,16 @@ def compare_scores(wl, conf, token, state_out, w_out=None, counts=None, cur_toke
                 assert token[r] == res.token[i], (si, i, token[r], res.token[i])
                 if tokens_next is not None:
                     assert tokens_next[r] == res.tokens_next[i], (si, i, tokens_next[r])
+            if entropy is not None:
+                herr = abs(float(entropy[r]) - res.entropy[i])
+                rep["max_entropy_err"] = max(rep.get("max_entropy_err", 0.0), herr)
+                assert herr <= ENTROPY_TOL, (si, i, entropy[r], res.entropy[i])
+            if margin is not None:
+                assert abs(float(margin[r]) - res.margin[i]) <= CONF_TOL, (si, i, margin[r], res.margin[i])
+            if order_key is not None:
+                want = orc.order_key(order_mode, res.conf[i], res.entropy[i], res.margin[i], i)
+                tol = ENTROPY_TOL if order_mode == orc.ORDER_ENTROPY else CONF_TOL
+                assert abs(float(order_key[r]) - want) <= tol, (si, i, order_key[r], want)
             if p_cur is not None:
                 perr = abs(float(p_cur[r]) - res.p_cur[i])
                 rep["max_p_cur_err"] = max(rep.get("max_p_cur_err", 0.0), perr)

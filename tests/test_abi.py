@@ -114,7 +114,7 @@ def _score_args(**kw):
     ({"lambda_": 0.0}, 3), ({"p0": 0.0}, 3), ({"num_seqs": 0}, 2),
     ({"bl": np.array([200], np.int32)}, 2), ({"workspace": None}, 7),
     ({"workspace_bytes": 16}, 7), ({"logits_x": 0x10002}, 6), ({"row_stride": 1025}, 6),
-    ({"p_cur": 0x50000}, 1),
+    ({"p_cur": 0x50000}, 1), ({"order_mode": 5}, 3), ({"order_mode": -1}, 3),
 ])
 def test_score_validation(lib, change, code):
     a, keep = _score_args(**change)

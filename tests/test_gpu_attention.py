@@ -188,3 +188,19 @@ def test_attention_random_query_start(case, tc):
     offs = wl.row_offsets()
     for si, s in enumerate(wl.seqs):
         assert np.all(o[offs[si]:offs[si] + s.query_start] == 7.0)
+
+
+@pytest.mark.parametrize("mode", ["bidir", "l2r"])
+def test_attention_ordering_keys(mode, tc):
+    """The ablation's orderings enter the mask as the Eq. 3 key in prev_conf: equal keys
+    (every C pair mutual) and minus the block position (left-to-right among C). Uniform
+    attention (Q = 0) exposes every key selection."""
+    B = 64
+    rng = np.random.default_rng(3 if mode == "bidir" else 4)
+    st = rng.choice(np.array([0, 1, 2], np.uint8), size=B, p=[0.3, 0.5, 0.2])
+    key = np.zeros(B, np.float32) if mode == "bidir" else -np.arange(B, dtype=np.float32)
+    specs = [dict(n_orig=300, block_start=150, state=st, prev_conf=key)]
+    wl = W.custom(specs, 2, 2, 128, probe=True, seed=9)
+    _, o = _attend(wl)
+    mx, _, _ = P.compare_attention(wl, 0, o)
+    assert mx <= _probe_tol(wl)

@@ -151,3 +151,27 @@ def test_score_end_of_step(name, in_place):
                            p_cur=p_cur, tokens_next=tokens, mask_token=mask_token)
     assert int(ds.status.item()) == 0
     print(name, in_place, rep)
+
+
+@pytest.mark.parametrize("name", ["tiny", "8b", "gqa", "mm"])
+@pytest.mark.parametrize("mode", [B.ORDER_CONFIDENCE, B.ORDER_BIDIR, B.ORDER_L2R,
+                                  B.ORDER_ENTROPY, B.ORDER_MARGIN])
+def test_score_ordering_outputs(name, mode):
+    """Entropy and margin of every scored distribution, and the next step's ordering key
+    (the ablation's orderings: confidence, bidirectional, left-to-right, entropy, margin)."""
+    wl = W.make(name, logits="spanning", attention=False)
+    ds = DeviceStep(wl, attention=False)
+    rows = ds.state.numel()
+    dev = ds.state.device
+    ent, mg, key = (torch.full((rows,), 99.0, dtype=torch.float32, device=dev) for _ in range(3))
+    B.dard_score_and_transition(ds.lx, ds.ls, ds.block_len, ds.state, wl.tau_c, wl.tau_u, wl.lam,
+                                wl.p0, ds.conf, ds.token, ds.state_out, ds.workspace,
+                                w_out=ds.w_out, counts=ds.counts, status=ds.status, entropy=ent,
+                                margin=mg, order_key=key, order_mode=mode)
+    torch.cuda.synchronize()
+    out = [t.cpu().numpy() for t in (ds.conf, ds.token, ds.state_out, ds.w_out, ds.counts,
+                                     ent, mg, key)]
+    rep = P.compare_scores(wl, *out[:3], w_out=out[3], counts=out[4], entropy=out[5],
+                           margin=out[6], order_key=out[7], order_mode=mode)
+    assert int(ds.status.item()) == 0
+    print(name, mode, rep)
