@@ -217,52 +217,40 @@ __device__ __forceinline__ int load_state(const ScoreParams& p, int row, bool re
   return s;
 }
 
-// ---- the extended summary of the end-of-step variant: also the entropy sum
-// h = sum exp(x - m) (x - m) and the second-largest value m2 (a repeated maximum counts as
-// the second), for the entropy and the margin of the ordering variants.
+// ---- the extended summary of the end-of-step variant: also hx = sum exp(x - m) x (the
+// entropy sum is h = sum exp(x - m)(x - m) = hx - m s) and the second-largest value m2 (a
+// repeated maximum counts as the second), for the entropy and margin of the ordering
+// variants. Both rescale like s when the maximum grows.
 struct AccX {
   float m;   // running maximum
   float s;   // sum of exp(x - m)
   int idx;   // lowest index attaining m
-  float h;   // sum of exp(x - m) * (x - m)
+  float hx;  // sum of exp(x - m) * x
   float m2;  // second-largest value
 };
 
 __device__ __forceinline__ AccX accx_init() { return {-INFINITY, 0.f, INT_MAX, 0.f, -INFINITY}; }
 
-// Re-expresses (s, h) of maximum m_old against the larger maximum m_new.
-__device__ __forceinline__ void accx_rescale(float& s, float& h, float m_old, float m_new) {
-  if (m_old == -INFINITY) {
-    s = 0.f;
-    h = 0.f;
-    return;
-  }
-  const float d = m_old - m_new;  // <= 0
-  const float f = ex2_approx(d * kLog2e);
-  h = f * fmaf(d, s, h);
-  s = s * f;
-}
-
-__device__ __forceinline__ AccX accx_merge(const AccX& a, const AccX& b) {
-  const bool b_wins = (b.m > a.m) || (b.m == a.m && b.idx < a.idx);
-  const AccX hi = b_wins ? b : a;
-  AccX lo = b_wins ? a : b;
-  accx_rescale(lo.s, lo.h, lo.m, hi.m);
-  return {hi.m, hi.s + lo.s, hi.idx, hi.h + lo.h, fmaxf(fmaxf(a.m2, b.m2), lo.m)};
-}
-
-__device__ __forceinline__ AccX warp_merge(AccX a) {
+// Warp-wide merge in the manner of warp_merge_fast; the second maximum is the largest of
+// every lane's second value and of the first values of the lanes that do not hold the
+// winning (maximum, lowest index) entry.
+__device__ __forceinline__ AccX warp_merge_fast(const AccX& a) {
+  const uint32_t key = order_key(a.m);
+  const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+  const float mx = from_key(kmax);
+  const uint32_t cand = key == kmax ? static_cast<uint32_t>(a.idx) : 0xffffffffu;
+  const int idx = static_cast<int>(__reduce_min_sync(0xffffffffu, cand));
+  const bool winner = key == kmax && a.idx == idx;
+  const float c2 = winner ? a.m2 : fmaxf(a.m, a.m2);
+  const float m2 = from_key(__reduce_max_sync(0xffffffffu, order_key(c2)));
+  const float f = (a.m == -INFINITY) ? 0.f : ex2_approx((a.m - mx) * kLog2e);
+  float sum = a.s * f, hx = a.hx * f;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
-    AccX b;
-    b.m = __shfl_xor_sync(0xffffffffu, a.m, off);
-    b.s = __shfl_xor_sync(0xffffffffu, a.s, off);
-    b.idx = __shfl_xor_sync(0xffffffffu, a.idx, off);
-    b.h = __shfl_xor_sync(0xffffffffu, a.h, off);
-    b.m2 = __shfl_xor_sync(0xffffffffu, a.m2, off);
-    a = accx_merge(a, b);
+    sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    hx += __shfl_xor_sync(0xffffffffu, hx, off);
   }
-  return a;
+  return {mx, sum, idx, hx, m2};
 }
 
 template <class T, int VPT, bool kTail, class ValFn>
@@ -280,25 +268,24 @@ __device__ __forceinline__ void fold_round(AccX& acc, int base, int limit, ValFn
 #pragma unroll
     for (int e = 0; e < T::W; ++e) {
       const float x = get(v, e);
+      m2 = fmaxf(m2, fminf(x, m));  // the old maximum, or x, becomes a second candidate
       if (x > m) {
-        m2 = m;
         m = x;
         idx = base + (v * kScoreThreads + static_cast<int>(threadIdx.x)) * T::W + e;
-      } else {
-        m2 = fmaxf(m2, x);
       }
     }
   }
-  const float m2_all = fmaxf(fmaxf(acc.m2, m2), fminf(acc.m, m));
+  acc.m2 = fmaxf(fmaxf(acc.m2, m2), fminf(acc.m, m));
   if (m > acc.m) {
-    accx_rescale(acc.s, acc.h, acc.m, m);
+    const float f = (acc.m == -INFINITY) ? 0.f : ex2_approx((acc.m - m) * kLog2e);
+    acc.s *= f;
+    acc.hx *= f;
     acc.m = m;
     acc.idx = idx;
   }
-  acc.m2 = m2_all;
   if (acc.m == -INFINITY) return;
   const float mL = acc.m * kLog2e;
-  float s = 0.f, h = 0.f;
+  float s = 0.f, hx = 0.f;
 #pragma unroll
   for (int v = 0; v < VPT; ++v) {
 #pragma unroll
@@ -306,11 +293,11 @@ __device__ __forceinline__ void fold_round(AccX& acc, int base, int limit, ValFn
       const float x = get(v, e);
       const float ex = ex2_approx(fmaf(x, kLog2e, -mL));
       s += ex;
-      h = fmaf(ex, fmaxf(x - acc.m, -1e30f), h);  // -inf elements add 0, not NaN
+      hx = fmaf(ex, fmaxf(x, -FLT_MAX), hx);  // -inf elements add 0, not NaN
     }
   }
   acc.s += s;
-  acc.h += h;
+  acc.hx += hx;
 }
 
 template <class T, int VPT, class ValFn>
@@ -320,13 +307,13 @@ __device__ __forceinline__ void fold(AccX& acc, int base, int limit, ValFn val) 
 }
 
 __device__ __forceinline__ AccX block_merge(AccX a, AccX* smem) {
-  a = warp_merge(a);
+  a = warp_merge_fast(a);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (lane == 0) smem[warp] = a;
   __syncthreads();
   if (warp == 0) {
     a = lane < kWarps ? smem[lane] : accx_init();
-    a = warp_merge(a);
+    a = warp_merge_fast(a);
   }
   return a;  // valid in warp 0
 }
@@ -343,7 +330,7 @@ __device__ __forceinline__ void cluster_publish(const Acc& a, int split, float4*
 __device__ __forceinline__ void cluster_publish(const AccX& a, int split, float4* slots) {
   if (threadIdx.x == 0) {
     st_cluster_v4(map_shared_rank(smem_u32(&slots[split]), 0), a.m, a.s, __int_as_float(a.idx),
-                  a.h);
+                  a.hx);
     st_cluster_v4(map_shared_rank(smem_u32(&slots[kScoreMaxSplit + split]), 0), a.m2, 0.f, 0.f,
                   0.f);
   }
@@ -367,19 +354,24 @@ __device__ __forceinline__ void merge_slots(const float4* slots, int nsplit, Acc
     const float4 v = slots[lane], v2 = slots[kScoreMaxSplit + lane];
     a = AccX{v.x, v.y, __float_as_int(v.z), v.w, v2.x};
   }
-  out = warp_merge(a);
+  out = warp_merge_fast(a);
 }
 
 __device__ __forceinline__ Acc acc_init(Acc*) { return {-INFINITY, 0.f, INT_MAX}; }
 __device__ __forceinline__ AccX acc_init(AccX*) { return accx_init(); }
 
-// The scored logit of the current token (p_cur), or NaN without one. lf(col) returns the
-// row's scored logit at col (shadow, or mixed for M rows).
-template <class LogitFn>
-__device__ __forceinline__ float current_logit(const ScoreParams& p, int row, LogitFn lf) {
-  if (p.p_cur == nullptr) return __int_as_float(0x7fc00000);
+// The current token's logits (for p_cur), loaded by the leader's thread 0 when the CTA
+// starts so that their latency hides behind the row's stream; -inf marks "no token".
+template <class T>
+__device__ __forceinline__ void prefetch_current(const ScoreParams& p, int row, const char* xp,
+                                                 const char* sp, float& lx, float& ls) {
+  lx = ls = -INFINITY;
+  if (p.p_cur == nullptr || threadIdx.x != 0 || blockIdx.x != 0) return;
   const int ct = p.cur_token[row];
-  return (ct >= 0 && ct < p.vocab) ? lf(ct) : -INFINITY;
+  if (ct < 0 || ct >= p.vocab) return;
+  const size_t off = static_cast<size_t>(ct) * T::kBytes;
+  ls = T::scalar(sp + off);
+  if (xp) lx = T::scalar(xp + off);
 }
 
 // Eq. 1 and Eq. 8 on a merged row; writes conf / token / state, the optional p_cur (of the
@@ -403,7 +395,7 @@ __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const
   if (kExtra && p.tokens) p.tokens[row] = ns == kStateM ? p.mask_token : a.idx;
   if constexpr (kExtra) {
     // entropy (nats) and margin of the scored distribution, the next step's ordering key
-    const float hnat = valid ? logf(z) - a.h / z : 0.f;
+    const float hnat = valid ? logf(z) + a.m - a.hx / z : 0.f;  // ln Z - (hx - m Z) / Z
     const float mg = valid ? (1.0f - ex2_approx((a.m2 - a.m) * kLog2e)) / z : 0.f;
     if (p.entropy) p.entropy[row] = hnat;
     if (p.margin) p.margin[row] = mg;
@@ -446,6 +438,8 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   const char* rowp = static_cast<const char*>(p.ls) + static_cast<size_t>(row) * p.row_stride * T::kBytes;
   const int c0 = split * p.chunk;
   const int c1 = min(p.vocab, c0 + p.chunk);
+  float cur_lx = 0.f, cur_ls = 0.f;  // the current token's logit (p_cur), loaded early
+  if (kExtra) prefetch_current<T>(p, row, nullptr, rowp, cur_lx, cur_ls);
   A acc = acc_init(static_cast<A*>(nullptr));
   for (int base = c0; base < c1; base += kScoreThreads * VPT * T::W) {
     uint4 r[VPT];
@@ -460,10 +454,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_consta
   A a;
   merge_slots(s_slots, p.nsplit, a);
   if (threadIdx.x == 0) {
-    const float lc = !kExtra ? 0.f : current_logit(p, row, [&](int col) {
-      return T::scalar(rowp + static_cast<size_t>(col) * T::kBytes);
-    });
-    const int ns = finalize_row<kExtra>(p, row, a, __int_as_float(0x7fc00000), lc);
+    const int ns = finalize_row<kExtra>(p, row, a, __int_as_float(0x7fc00000), cur_ls);
     p.pd_flag[row] = (st == kStateC) ? (ns == kStateU ? 1 : (ns == kStateM ? 2 : 0)) : 0;
   }
 }
@@ -490,6 +481,8 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   const char* sp = static_cast<const char*>(p.ls) + roff;
   const int c0 = split * p.chunk;
   const int c1 = min(p.vocab, c0 + p.chunk);
+  float cur_lx = 0.f, cur_ls = 0.f;  // the current token's logits (p_cur), loaded early
+  if (kExtra) prefetch_current<T>(p, row, xp, sp, cur_lx, cur_ls);
 
   // The first round's loads do not depend on pass 1: issue them before waiting for it.
   uint4 rx[VPT], rs[VPT];
@@ -557,11 +550,8 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   A a;
   merge_slots(s_slots, p.nsplit, a);
   if (threadIdx.x == 0) {
-    const float lc = !kExtra ? 0.f : current_logit(p, row, [&](int col) {
-      const size_t off = static_cast<size_t>(col) * T::kBytes;
-      const float lx = T::scalar(xp + off), ls = T::scalar(sp + off);
-      return __fadd_rn(ls, __fmul_rn(w, __fsub_rn(lx, ls)));
-    });
+    const float lc = cur_ls == -INFINITY ? -INFINITY
+                                         : __fadd_rn(cur_ls, __fmul_rn(w, __fsub_rn(cur_lx, cur_ls)));
     add_count(p, seq, finalize_row<kExtra>(p, row, a, w, lc));
   }
 }
