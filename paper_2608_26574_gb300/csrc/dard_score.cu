@@ -425,6 +425,10 @@ __device__ __forceinline__ void add_count(const ScoreParams& p, int seq, int sta
 template <class T, int VPT, bool kExtra>
 __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_constant__ ScoreParams p) {
   grid_dep_launch();  // pass 2 may start loading its logits right away
+  // Launched with programmatic dependent launch after whatever kernel precedes the call
+  // (the LM head in a model, the attention kernel in the benchmark): this CTA may already be
+  // resident, but it touches no memory before that kernel has completed.
+  grid_dep_wait();
   using A = std::conditional_t<kExtra, AccX, Acc>;
   __shared__ A s_acc[kWarps];
   __shared__ float4 s_slots[2 * kScoreMaxSplit];
@@ -592,7 +596,7 @@ cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   e = cudaLaunchKernelEx(&cfg, score_pass1<T, VPT, kExtra>, p);
   if (e != cudaSuccess) return e;
   cfg.numAttrs = 2;
