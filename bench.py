@@ -153,6 +153,18 @@ def traffic_for(kernel: str, source: str, per_launch_units: float):
     return None
 
 
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The largest value of x over all ranks (every rank gets it); x itself with one rank.
+    Works with NCCL (device tensor) and gloo (host tensor)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def oracle_step(wl, rows=None):
     """One oracle pass over the workload's first sequence: mask + attention (all heads) for
     `rows` query rows (all when None) and scoring of the whole block. Returns
@@ -325,10 +337,7 @@ def run_ours(args, rank: int, world: int):
     if world > 1:
         dist.barrier()
     clocks = mon.stop()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, dev)
     ms_per_step = ms / args.steps
 
     # per-kernel averages (same launches, one kernel per graph)
