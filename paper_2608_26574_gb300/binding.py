@@ -113,9 +113,14 @@ def _rows_ptr(t) -> int:
     """Device pointer of a 2-D tensor whose rows are contiguous (any row pitch)."""
     if not t.is_cuda:
         raise ValueError("device tensor expected")
-    if t.dim() != 2 or t.stride(1) != 1:
+    if t.dim() != 2 or (t.numel() > 0 and t.stride(1) != 1):
         raise ValueError("2-D tensor with contiguous rows expected")
     return t.data_ptr()
+
+
+def _row_pitch(t) -> int:
+    """Elements between rows (an empty tensor has no rows to step over: its width)."""
+    return t.stride(0) if t.numel() > 0 else t.shape[1]
 
 
 def _host_i32(a) -> np.ndarray:
@@ -175,13 +180,13 @@ def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, ta
     ``p_cur`` of ``cur_token``, and ``tokens`` (x^, or ``mask_token`` for rows ending in M);
     ``entropy``, ``margin`` and the next step's ``order_key`` for ``order_mode``."""
     block_len = _host_i32(block_len)
-    if logits_x.stride(0) != logits_s.stride(0) or logits_x.shape != logits_s.shape:
+    if _row_pitch(logits_x) != _row_pitch(logits_s) or logits_x.shape != logits_s.shape:
         raise ValueError("logits_x and logits_s need the same shape and row pitch")
     a = ScoreArgs()
     a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
     a.dtype = _dtype_code(logits_s)
     a.vocab = logits_s.shape[1]
-    a.row_stride = logits_s.stride(0)
+    a.row_stride = _row_pitch(logits_s)
     a.num_seqs = len(block_len)
     a.block_len = block_len.ctypes.data_as(_I32P)
     a.state_in = _ptr(state_in)
@@ -204,13 +209,13 @@ def dard_score_and_transition_noalloc(logits_x, logits_s, block_len, state_in, t
     """``dard_score_and_transition`` without a workspace: the library's built-in scratch
     (at most ``SCORE_NOALLOC_MAX_ROWS`` block rows; calls that overlap on one device race)."""
     block_len = _host_i32(block_len)
-    if logits_x.stride(0) != logits_s.stride(0) or logits_x.shape != logits_s.shape:
+    if _row_pitch(logits_x) != _row_pitch(logits_s) or logits_x.shape != logits_s.shape:
         raise ValueError("logits_x and logits_s need the same shape and row pitch")
     a = ScoreArgs()
     a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
     a.dtype = _dtype_code(logits_s)
     a.vocab = logits_s.shape[1]
-    a.row_stride = logits_s.stride(0)
+    a.row_stride = _row_pitch(logits_s)
     a.num_seqs = len(block_len)
     a.block_len = block_len.ctypes.data_as(_I32P)
     a.state_in = _ptr(state_in)

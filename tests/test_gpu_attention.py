@@ -204,3 +204,32 @@ def test_attention_ordering_keys(mode, tc):
     _, o = _attend(wl)
     mx, _, _ = P.compare_attention(wl, 0, o)
     assert mx <= _probe_tol(wl)
+
+
+def test_attention_maximum_batch(tc):
+    """DARD_MAX_SEQS sequences with full 128-position blocks and their shadow rows."""
+    rng = np.random.default_rng(91)
+    specs = []
+    for _ in range(256):
+        n = int(rng.integers(128, 300))
+        b0 = int(rng.integers(0, n - 128 + 1))
+        specs.append(dict(n_orig=n, block_start=b0, block_len=128,
+                          fractions=tuple(rng.dirichlet([1, 1, 1]))))
+    wl = W.custom(specs, 2, 1, 64, seed=92)
+    ds, o = _attend(wl)
+    # a sample of rows per sequence, every block and shadow row of a few sequences
+    mx, mean, n = P.compare_attention(wl, 0, o, sample=8)
+    assert mx <= P.att_tol(wl) and mean <= P.ATT_MEAN_ABS
+    assert int(ds.status.item()) == 0
+
+
+def test_attention_no_query_rows(tc):
+    """query_start at the end of every sequence: nothing is launched, the output is untouched."""
+    specs = [dict(n_orig=90, block_start=10, block_len=16, fractions=(0.3, 0.4, 0.3),
+                  query_start=106) for _ in range(2)]
+    wl = W.custom(specs, 2, 2, 128, seed=93)
+    ds = DeviceStep(wl, layers=[0], scoring=False)
+    out = _sentinel_out(ds)
+    ds.attention(0, out=out)
+    torch.cuda.synchronize()
+    assert bool((out == 7.0).all())

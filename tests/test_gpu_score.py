@@ -175,3 +175,25 @@ def test_score_ordering_outputs(name, mode):
                            margin=out[6], order_key=out[7], order_mode=mode)
     assert int(ds.status.item()) == 0
     print(name, mode, rep)
+
+
+def test_score_maximum_batch():
+    """The largest call the ABI allows: DARD_MAX_SEQS sequences with blocks of
+    DARD_MAX_BLOCK positions (32768 rows), a small vocabulary."""
+    specs = [dict(n_orig=B.MAX_BLOCK + 3, block_start=2, block_len=B.MAX_BLOCK,
+                  fractions=(0.4, 0.3, 0.3)) for _ in range(B.MAX_SEQS)]
+    wl = W.custom(specs, 1, 1, 64, vocab=256, seed=77, logit_std=2.0)
+    ds, outs = _run(wl)
+    _check(wl, outs)
+    assert int(ds.status.item()) == 0
+
+
+def test_score_all_blocks_empty():
+    """Every block empty: no pass runs, and the counts still come out as zeros."""
+    specs = [dict(n_orig=40, block_start=5, block_len=0, fractions=(1, 0, 0)) for _ in range(3)]
+    wl = W.custom(specs, 1, 1, 64, vocab=512, seed=1)
+    ds = DeviceStep(wl, attention=False)
+    ds.counts.fill_(-5)
+    ds.score()
+    torch.cuda.synchronize()
+    assert ds.counts.cpu().tolist() == [0] * 9
