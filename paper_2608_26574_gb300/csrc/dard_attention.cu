@@ -8,22 +8,31 @@
 // so the mask is evaluated only on the (at most three) tiles that contain block keys,
 // shadow keys or the ragged end of the sequence.
 //
-// bf16 path (attn_tc): one CTA per SM = 128 query rows of one (sequence, head); 11 warps:
+// bf16 paths (tcgen05 MMAs with fp32 accumulators in TMEM, K/V tiles of 128 keys by TMA),
+// one CTA per SM, chosen per call by a cost model (launch_tc):
+//
+// attn_tc1: 128 query rows of one (sequence, head); 11 warps:
 //   warps 0-7  softmax and epilogue: warps w and w + 4 share TMEM lane quarter w (query
 //              rows 32w .. 32w + 31), each taking 64 of a tile's 128 key columns;
-//   warp 8     TMA producer: K and V tiles of 128 keys through 3 stages each, with L2
-//              prefetches a few tiles further ahead;
-//   warp 9     TMEM allocator and PV issuer: O += P_j V_j with P_j (bf16) read from TMEM,
-//              where the softmax warps wrote it over the first half of each warp's S_j
-//              columns;
-//   warp 10    S issuer: S_j = Q K_j^T (tcgen05, Q from TMEM, K from shared memory) into a
-//              ring of two 128-column TMEM buffers, each reused once the PV that reads the
-//              P stored in it has completed.
-// The softmax threads write their query rows into TMEM (bf16 pairs, the A-operand layout)
-// at the start, so shared-memory bandwidth goes to K and V only. With P in its own S
-// buffer, the softmax of tile j + 1 never waits for the PV of tile j.
-// The online softmax keeps a per-row running maximum and rescales O in TMEM only when the
-// maximum grows by more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
+//   warp 8     TMA producer: K and V through 3 stages each, L2 prefetches further ahead;
+//   warp 9     TMEM allocator and PV issuer: O += P_j V_j, P_j (bf16) read from TMEM;
+//   warp 10    S issuer: S_j = Q K_j^T (Q from TMEM, K from shared memory) into a ring of
+//              two 128-column TMEM buffers, reused once the softmax has read S_j.
+//   TMEM: S ring [0, 256), O [256, 256 + D), P [384, 448), Q [448, 448 + D/2). The
+//   softmax threads write their query rows into TMEM at the start, so shared-memory
+//   bandwidth goes to K and V only.
+//
+// attn_tc2: two 128-row query tiles of the same (sequence, head), so that every K/V tile
+// serves 256 rows; 10 warps:
+//   warps 4q .. 4q + 3  softmax and epilogue of tile q, one thread per query row;
+//   warp 8              TMA producer: both Q tiles, then K and V through 2 stages each;
+//   warp 9              TMEM allocator and MMA issuer, in the order S_0(0) S_1(0) |
+//                       PV_0(j) S_0(j+1) PV_1(j) S_1(j+1) | ... (Q from shared memory).
+//   TMEM: S_0, S_1 [0, 256) with P_q(j) written over the first 64 columns of S_q(j),
+//   O_0, O_1 [256, 256 + 2D). S_q(j+1) is issued once PV_q(j) has read P_q(j).
+//
+// Both keep a per-row running maximum and rescale O in TMEM only when the maximum grows by
+// more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
 // fp32 path (attn_simt): CUDA-core kernel, one warp per query row, same mask logic.
 #include <cuda.h>
 #include <cuda_bf16.h>

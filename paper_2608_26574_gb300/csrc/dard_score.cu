@@ -15,7 +15,12 @@
 // CTA over DSMEM; after one cluster barrier that CTA merges the partials in split order
 // (deterministic) and writes the row's outputs. Pass 2 is launched as a programmatic
 // dependent of pass 1: its CTAs load their logits while pass 1 finishes and only then
-// wait for pass 1's results.
+// wait for pass 1's results. Pass 1 is itself a programmatic dependent of whatever kernel
+// precedes the call and waits for it before touching memory.
+//
+// The number of CTAs per row follows the row count (split_cap). A compile-time variant
+// (kExtra) adds the optional end-of-step outputs: p_cur, the next step's tokens, an
+// in-place state update, entropy, margin and the next step's ordering key.
 #include <atomic>
 #include <type_traits>
 #include <cfloat>
