@@ -99,13 +99,58 @@ def _check(code: int, fn: str):
         raise DardError(code, fn, lib().dard_last_error().decode())
 
 
-def _ptr(t) -> int | None:
+def _host_i32(a) -> np.ndarray:
+    """An owned, contiguous int32 copy of a per-sequence host array."""
+    return np.array(a, dtype=np.int32, copy=True).reshape(-1)
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _raw_stream(device_index: int) -> int:
+    """cudaStream_t of the device's current torch stream."""
+    torch = _torch()
+    f = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+    if f is not None:
+        return f(device_index)
+    return torch.cuda.current_stream(device_index).cuda_stream
+
+
+def _stream_handle(stream, device_index: int) -> int:
+    """``stream`` as a raw handle: a torch stream, an int, or None for the current stream."""
+    if stream is None:
+        return _raw_stream(device_index)
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _dtype_code(t) -> int:
+    torch = _torch()
+    if t.dtype == torch.bfloat16:
+        return DARD_BF16
+    if t.dtype == torch.float32:
+        return DARD_F32
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def _dev(t, name: str, n: int, dtype, device: int | None = None) -> int | None:
+    """Device pointer of an optional contiguous tensor of ``dtype`` with at least ``n``
+    elements (None for a missing tensor)."""
     if t is None:
         return None
     if not t.is_cuda:
-        raise ValueError("device tensor expected")
+        raise ValueError(f"{name}: device tensor expected")
     if not t.is_contiguous():
-        raise ValueError("contiguous tensor expected")
+        raise ValueError(f"{name}: contiguous tensor expected")
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: {dtype} expected, got {t.dtype}")
+    if t.numel() < n:
+        raise ValueError(f"{name}: at least {n} elements expected, got {t.numel()}")
+    if device is not None and t.get_device() != device:
+        raise ValueError(f"{name}: on device {t.get_device()}, expected {device}")
     return t.data_ptr()
 
 
@@ -123,23 +168,69 @@ def _row_pitch(t) -> int:
     return t.stride(0) if t.numel() > 0 else t.shape[1]
 
 
-def _host_i32(a) -> np.ndarray:
-    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+class AttentionCall:
+    """``dard_step_attention`` with everything but q, k, v and o marshalled once.
 
+    One step's per-sequence metadata and mask inputs (states, c_{t-1}, shadow sources) are
+    the same for every layer, so a caller running many layers builds this once per step and
+    calls it per layer. The host arrays are copied; the device tensors are referenced and
+    must stay alive and unchanged in size while the object is used. Each call checks q, k,
+    v and o against the row count the metadata implies (sum of n_orig + shadow_len), sets
+    the four pointers and the stream, and calls the library."""
 
-def _stream(stream) -> int:
-    import torch
-    s = stream if stream is not None else torch.cuda.current_stream()
-    return s.cuda_stream
+    def __init__(self, n_orig, block_start, block_len, shadow_len, state, prev_conf,
+                 shadow_src, scale: float = 0.0, status=None, query_start=None):
+        torch = _torch()
+        self._host = [_host_i32(x) for x in (n_orig, block_start, block_len, shadow_len)]
+        self._qs = _host_i32(query_start) if query_start is not None else None
+        n, b0, bl, sl = self._host
+        ns = len(n)
+        if any(len(x) != ns for x in self._host[1:]) or (self._qs is not None and
+                                                        len(self._qs) != ns):
+            raise ValueError("per-sequence arrays differ in length")
+        self.rows = int(n.astype(np.int64).sum() + sl.astype(np.int64).sum())
+        blk, sh = int(bl.astype(np.int64).sum()), int(sl.astype(np.int64).sum())
+        self.device = state.get_device() if state is not None else None
+        a = AttnArgs()
+        a.num_seqs = ns
+        a.n_orig, a.block_start, a.block_len, a.shadow_len = (
+            x.ctypes.data_as(_I32P) for x in self._host)
+        a.query_start = self._qs.ctypes.data_as(_I32P) if self._qs is not None else None
+        a.state = _dev(state, "state", blk, torch.uint8)
+        a.prev_conf = _dev(prev_conf, "prev_conf", blk, torch.float32, self.device)
+        a.shadow_src = _dev(shadow_src, "shadow_src", sh, torch.int32, self.device)
+        a.status = _dev(status, "status", 1, torch.int32, self.device)
+        a.scale = scale
+        self._keep = (state, prev_conf, shadow_src, status)
+        self._args = a
+        self._ref = ctypes.byref(a)
+        self._fn = lib().dard_step_attention
 
-
-def _dtype_code(t) -> int:
-    import torch
-    if t.dtype == torch.bfloat16:
-        return DARD_BF16
-    if t.dtype == torch.float32:
-        return DARD_F32
-    raise ValueError(f"unsupported dtype {t.dtype}")
+    def __call__(self, q, k, v, o, stream=None):
+        """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d]."""
+        if not (q.is_cuda and k.is_cuda and v.is_cuda and o.is_cuda):
+            raise ValueError("q, k, v and o must be device tensors")
+        if not (q.is_contiguous() and k.is_contiguous() and v.is_contiguous()
+                and o.is_contiguous()):
+            raise ValueError("q, k, v and o must be contiguous")
+        qs, ks = q.shape, k.shape
+        if (len(qs) != 3 or len(ks) != 3 or o.shape != qs or v.shape != ks or ks[2] != qs[2]
+                or qs[0] < self.rows or ks[0] < self.rows):
+            raise ValueError(f"q/o [>={self.rows}, hq, d] and k/v [>={self.rows}, hkv, d] "
+                             f"expected, got {tuple(qs)}, {tuple(ks)}, {tuple(v.shape)}, "
+                             f"{tuple(o.shape)}")
+        dt = q.dtype
+        if k.dtype != dt or v.dtype != dt or o.dtype != dt:
+            raise ValueError("q, k, v and o need one dtype")
+        dev = q.get_device()
+        if (k.get_device() != dev or v.get_device() != dev or o.get_device() != dev
+                or (self.device is not None and dev != self.device)):
+            raise ValueError("q, k, v, o and the mask inputs need one device")
+        a = self._args
+        a.q, a.k, a.v, a.o = q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr()
+        a.dtype = _dtype_code(q)
+        a.hq, a.hkv, a.head_dim = qs[1], ks[1], qs[2]
+        _check(self._fn(self._ref, _stream_handle(stream, dev)), "dard_step_attention")
 
 
 def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, state,
@@ -147,27 +238,84 @@ def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, 
                         query_start=None):
     """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d] on the device.
     ``query_start`` (per sequence, optional): first query row; earlier rows are keys only."""
-    n_orig, block_start = _host_i32(n_orig), _host_i32(block_start)
-    qs = _host_i32(query_start) if query_start is not None else None
-    block_len, shadow_len = _host_i32(block_len), _host_i32(shadow_len)
-    a = AttnArgs()
-    a.q, a.k, a.v, a.o = _ptr(q), _ptr(k), _ptr(v), _ptr(o)
-    a.dtype = _dtype_code(q)
-    a.hq, a.hkv, a.head_dim = q.shape[1], k.shape[1], q.shape[2]
-    a.num_seqs = len(n_orig)
-    a.n_orig = n_orig.ctypes.data_as(_I32P)
-    a.block_start = block_start.ctypes.data_as(_I32P)
-    a.block_len = block_len.ctypes.data_as(_I32P)
-    a.shadow_len = shadow_len.ctypes.data_as(_I32P)
-    a.state, a.prev_conf, a.shadow_src = _ptr(state), _ptr(prev_conf), _ptr(shadow_src)
-    a.scale = scale
-    a.status = _ptr(status)
-    a.query_start = qs.ctypes.data_as(_I32P) if qs is not None else None
-    _check(lib().dard_step_attention(ctypes.byref(a), _stream(stream)), "dard_step_attention")
+    AttentionCall(n_orig, block_start, block_len, shadow_len, state, prev_conf, shadow_src,
+                  scale=scale, status=status, query_start=query_start)(q, k, v, o, stream)
 
 
 def dard_score_workspace_size(rows: int, vocab: int, num_seqs: int) -> int:
     return int(lib().dard_score_workspace_size(rows, vocab, num_seqs))
+
+
+class ScoreCall:
+    """``dard_score_and_transition`` with everything but the two logits tensors marshalled
+    once: the block lengths, thresholds and every state and output buffer. A decode loop
+    builds it once per block (or once, with in-place states) and calls it each step on that
+    step's logits. The device tensors are referenced and must stay alive and unchanged in
+    size while the object is used. ``workspace=None`` selects
+    ``dard_score_and_transition_noalloc`` (the library's built-in scratch)."""
+
+    def __init__(self, block_len, state_in, tau_c, tau_u, lam, p0, conf, token, state_out,
+                 workspace, w_out=None, counts=None, status=None, cur_token=None, p_cur=None,
+                 tokens=None, mask_token: int = 0, entropy=None, margin=None, order_key=None,
+                 order_mode: int = ORDER_CONFIDENCE):
+        torch = _torch()
+        self._bl = _host_i32(block_len)
+        ns = len(self._bl)
+        self.rows = rows = int(self._bl.astype(np.int64).sum())
+        self.device = dev = state_in.get_device() if state_in is not None else None
+        f32, i32, u8 = torch.float32, torch.int32, torch.uint8
+        a = ScoreArgs()
+        a.num_seqs = ns
+        a.block_len = self._bl.ctypes.data_as(_I32P)
+        a.state_in = _dev(state_in, "state_in", rows, u8)
+        a.tau_c, a.tau_u, a.lambda_, a.p0 = tau_c, tau_u, lam, p0
+        a.conf = _dev(conf, "conf", rows, f32, dev)
+        a.token = _dev(token, "token", rows, i32, dev)
+        a.state_out = _dev(state_out, "state_out", rows, u8, dev)
+        a.w_out = _dev(w_out, "w_out", rows, f32, dev)
+        a.counts = _dev(counts, "counts", 3 * ns, i32, dev)
+        a.status = _dev(status, "status", 1, i32, dev)
+        a.cur_token = _dev(cur_token, "cur_token", rows, i32, dev)
+        a.p_cur = _dev(p_cur, "p_cur", rows, f32, dev)
+        a.tokens = _dev(tokens, "tokens", rows, i32, dev)
+        a.mask_token = mask_token
+        a.entropy = _dev(entropy, "entropy", rows, f32, dev)
+        a.margin = _dev(margin, "margin", rows, f32, dev)
+        a.order_key = _dev(order_key, "order_key", rows, f32, dev)
+        a.order_mode = order_mode
+        if workspace is not None:
+            a.workspace = _dev(workspace, "workspace", 0, workspace.dtype, dev)
+            a.workspace_bytes = workspace.numel() * workspace.element_size()
+            self._fn, self._name = lib().dard_score_and_transition, "dard_score_and_transition"
+        else:
+            self._fn = lib().dard_score_and_transition_noalloc
+            self._name = "dard_score_and_transition_noalloc"
+        self._keep = (state_in, conf, token, state_out, w_out, counts, status, cur_token,
+                      p_cur, tokens, entropy, margin, order_key, workspace)
+        self._args = a
+        self._ref = ctypes.byref(a)
+
+    def __call__(self, logits_x, logits_s, stream=None):
+        """Scores every block row; logits [rows, V] with contiguous rows and one row pitch
+        (``stride(0)``, at least V) in both tensors."""
+        shp = logits_s.shape
+        if logits_x.shape != shp or len(shp) != 2 or shp[0] < self.rows:
+            raise ValueError(f"logits_x and logits_s [>={self.rows}, V] of one shape expected, "
+                             f"got {tuple(logits_x.shape)} and {tuple(shp)}")
+        pitch = _row_pitch(logits_s)
+        if _row_pitch(logits_x) != pitch:
+            raise ValueError("logits_x and logits_s need the same row pitch")
+        if logits_x.dtype != logits_s.dtype:
+            raise ValueError("logits_x and logits_s need one dtype")
+        a = self._args
+        a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
+        dev = logits_s.get_device()
+        if logits_x.get_device() != dev or (self.device is not None and dev != self.device):
+            raise ValueError("the logits and the state and output buffers need one device")
+        a.dtype = _dtype_code(logits_s)
+        a.vocab = shp[1]
+        a.row_stride = pitch
+        _check(self._fn(self._ref, _stream_handle(stream, dev)), self._name)
 
 
 def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, tau_u, lam, p0,
@@ -179,28 +327,12 @@ def dard_score_and_transition(logits_x, logits_s, block_len, state_in, tau_c, ta
     the same row pitch (``stride(0)``, at least V) in both tensors. Optional end of step:
     ``p_cur`` of ``cur_token``, and ``tokens`` (x^, or ``mask_token`` for rows ending in M);
     ``entropy``, ``margin`` and the next step's ``order_key`` for ``order_mode``."""
-    block_len = _host_i32(block_len)
-    if _row_pitch(logits_x) != _row_pitch(logits_s) or logits_x.shape != logits_s.shape:
-        raise ValueError("logits_x and logits_s need the same shape and row pitch")
-    a = ScoreArgs()
-    a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
-    a.dtype = _dtype_code(logits_s)
-    a.vocab = logits_s.shape[1]
-    a.row_stride = _row_pitch(logits_s)
-    a.num_seqs = len(block_len)
-    a.block_len = block_len.ctypes.data_as(_I32P)
-    a.state_in = _ptr(state_in)
-    a.tau_c, a.tau_u, a.lambda_, a.p0 = tau_c, tau_u, lam, p0
-    a.conf, a.token, a.state_out = _ptr(conf), _ptr(token), _ptr(state_out)
-    a.w_out, a.counts, a.status = _ptr(w_out), _ptr(counts), _ptr(status)
-    a.workspace = _ptr(workspace)
-    a.workspace_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
-    a.cur_token, a.p_cur, a.tokens = _ptr(cur_token), _ptr(p_cur), _ptr(tokens)
-    a.mask_token = mask_token
-    a.entropy, a.margin, a.order_key = _ptr(entropy), _ptr(margin), _ptr(order_key)
-    a.order_mode = order_mode
-    _check(lib().dard_score_and_transition(ctypes.byref(a), _stream(stream)),
-           "dard_score_and_transition")
+    if workspace is None:
+        raise ValueError("workspace is required (see dard_score_workspace_size)")
+    ScoreCall(block_len, state_in, tau_c, tau_u, lam, p0, conf, token, state_out, workspace,
+              w_out=w_out, counts=counts, status=status, cur_token=cur_token, p_cur=p_cur,
+              tokens=tokens, mask_token=mask_token, entropy=entropy, margin=margin,
+              order_key=order_key, order_mode=order_mode)(logits_x, logits_s, stream)
 
 
 def dard_score_and_transition_noalloc(logits_x, logits_s, block_len, state_in, tau_c, tau_u,
@@ -208,19 +340,5 @@ def dard_score_and_transition_noalloc(logits_x, logits_s, block_len, state_in, t
                                       status=None, stream=None):
     """``dard_score_and_transition`` without a workspace: the library's built-in scratch
     (at most ``SCORE_NOALLOC_MAX_ROWS`` block rows; calls that overlap on one device race)."""
-    block_len = _host_i32(block_len)
-    if _row_pitch(logits_x) != _row_pitch(logits_s) or logits_x.shape != logits_s.shape:
-        raise ValueError("logits_x and logits_s need the same shape and row pitch")
-    a = ScoreArgs()
-    a.logits_x, a.logits_s = _rows_ptr(logits_x), _rows_ptr(logits_s)
-    a.dtype = _dtype_code(logits_s)
-    a.vocab = logits_s.shape[1]
-    a.row_stride = _row_pitch(logits_s)
-    a.num_seqs = len(block_len)
-    a.block_len = block_len.ctypes.data_as(_I32P)
-    a.state_in = _ptr(state_in)
-    a.tau_c, a.tau_u, a.lambda_, a.p0 = tau_c, tau_u, lam, p0
-    a.conf, a.token, a.state_out = _ptr(conf), _ptr(token), _ptr(state_out)
-    a.w_out, a.counts, a.status = _ptr(w_out), _ptr(counts), _ptr(status)
-    _check(lib().dard_score_and_transition_noalloc(ctypes.byref(a), _stream(stream)),
-           "dard_score_and_transition_noalloc")
+    ScoreCall(block_len, state_in, tau_c, tau_u, lam, p0, conf, token, state_out, None,
+              w_out=w_out, counts=counts, status=status)(logits_x, logits_s, stream)

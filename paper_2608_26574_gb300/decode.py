@@ -100,15 +100,17 @@ class DLLM:
         rows = batch.tokens.numel()
         h = self.emb[batch.tokens.long()]
         attn_outs = []
+        # one step's mask metadata serves every layer: marshalled once
+        attention = B.AttentionCall(batch.n_orig, batch.block_start, batch.block_len,
+                                    batch.shadow_len, batch.state, batch.prev_conf,
+                                    batch.shadow_src, status=batch.status)
         for L in self.layers:
             a = self.rmsnorm(h)
             q = self.rope((a @ L["wq"]).view(rows, cfg.hq, cfg.head_dim), batch.pos).contiguous()
             k = self.rope((a @ L["wk"]).view(rows, cfg.hkv, cfg.head_dim), batch.pos).contiguous()
             v = (a @ L["wv"]).view(rows, cfg.hkv, cfg.head_dim).contiguous()
             o = torch.empty_like(q)
-            B.dard_step_attention(q, k, v, o, batch.n_orig, batch.block_start, batch.block_len,
-                                  batch.shadow_len, batch.state, batch.prev_conf,
-                                  batch.shadow_src, status=batch.status)
+            attention(q, k, v, o)
             if need_attn_out:
                 attn_outs.append((q, k, v, o))
             h = h + o.view(rows, cfg.hq * cfg.head_dim) @ L["wo"]

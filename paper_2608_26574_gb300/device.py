@@ -38,6 +38,8 @@ class DeviceStep:
         sh = wl.shadow_src_all()
         self.shadow_src = torch.from_numpy(sh if len(sh) else np.zeros(1, np.int32)).to(dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self._attn_calls: dict[float, B.AttentionCall] = {}
+        self._score_calls: dict[tuple[bool, bool], B.ScoreCall] = {}
         self.layers = []
         if attention:
             idx = range(len(wl.q)) if layers is None else layers
@@ -67,18 +69,36 @@ class DeviceStep:
             self.w_out = torch.empty(r, dtype=torch.float32, device=dev)
             self.counts = torch.empty(3 * len(wl.seqs), dtype=torch.int32, device=dev)
 
+    def attention_call(self, scale: float = 0.0) -> B.AttentionCall:
+        """The prepared attention call of this step (metadata marshalled once per scale)."""
+        c = self._attn_calls.get(scale)
+        if c is None:
+            c = B.AttentionCall(self.n_orig, self.block_start, self.block_len, self.shadow_len,
+                                self.state, self.prev_conf, self.shadow_src, scale=scale,
+                                status=self.status, query_start=self.query_start)
+            self._attn_calls[scale] = c
+        return c
+
     def attention(self, layer: int = 0, scale: float = 0.0, stream=None, out=None):
         q, k, v, o = self.layers[layer]
-        B.dard_step_attention(q, k, v, o if out is None else out, self.n_orig, self.block_start,
-                              self.block_len, self.shadow_len, self.state, self.prev_conf,
-                              self.shadow_src, scale=scale, status=self.status, stream=stream,
-                              query_start=self.query_start)
-        return o if out is None else out
+        o = o if out is None else out
+        self.attention_call(scale)(q, k, v, o, stream)
+        return o
+
+    def score_call(self, w_out=True, counts=True, state_in=None) -> B.ScoreCall:
+        """The prepared scoring call over this step's buffers (cached for the step's own
+        states; a caller-given ``state_in`` gets a fresh one)."""
+        key = (bool(w_out), bool(counts))
+        c = self._score_calls.get(key) if state_in is None else None
+        if c is None:
+            wl = self.wl
+            c = B.ScoreCall(self.block_len, self.state if state_in is None else state_in,
+                            wl.tau_c, wl.tau_u, wl.lam, wl.p0, self.conf, self.token,
+                            self.state_out, self.workspace, w_out=self.w_out if w_out else None,
+                            counts=self.counts if counts else None, status=self.status)
+            if state_in is None:
+                self._score_calls[key] = c
+        return c
 
     def score(self, stream=None, w_out=True, counts=True, state_in=None):
-        wl = self.wl
-        B.dard_score_and_transition(
-            self.lx, self.ls, self.block_len, self.state if state_in is None else state_in,
-            wl.tau_c, wl.tau_u, wl.lam, wl.p0, self.conf, self.token, self.state_out,
-            self.workspace, w_out=self.w_out if w_out else None,
-            counts=self.counts if counts else None, status=self.status, stream=stream)
+        self.score_call(w_out, counts, state_in)(self.lx, self.ls, stream)
