@@ -10,9 +10,10 @@ current block 3, shadow copy of the current block (800 rows), logits 32 x 126464
 Timing: CUDA graphs of 16 consecutive steps, each on its own input set (16 sets, 675 MB,
 more than 4x the 129 MB L2), replayed back to back between CUDA events; per-kernel averages
 from graphs of the same 16 launches of one kernel. e2e: the same step through the C ABI
-from pinned host buffers, host->device copies of the inputs and device->host copies of the
-results inside the timed region (Q/K/V first, the logits on a second stream while the
-attention kernel runs; the ~0.2 TB/s host link bounds this number).
+from pinned host buffers, host->device copies of every input and device->host copies of the
+results inside the timed region, two steps in flight (step i + 1's inputs cross the host
+link, ~0.2 TB/s and the bound of this number, while step i computes); the one-step-at-a-time
+figure is reported beside it.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 """
@@ -346,48 +347,90 @@ def run_ours(args, rank: int, world: int):
     score_us = timed(g_score, reps) * 1e3 / (reps * NSETS)
     status = int(ds.status.item())
 
-    # e2e through the C ABI from pinned host buffers
-    host_in = {k: sets[0][k].cpu().pin_memory() for k in ("q", "k", "v", "lx", "ls")}
-    host_meta = {"state": ds.state.cpu().pin_memory(), "prev_conf": ds.prev_conf.cpu().pin_memory(),
-                 "shadow_src": ds.shadow_src.cpu().pin_memory()}
-    outs = {"conf": ds.conf, "token": ds.token, "state_out": ds.state_out, "counts": ds.counts}
-    host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in outs.items()}
-    d_meta = {"state": ds.state, "prev_conf": ds.prev_conf, "shadow_src": ds.shadow_src}
-    h2d = sum(t.numel() * t.element_size() for t in list(host_in.values()) + list(host_meta.values()))
-    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
-    s0 = sets[0]
+    # e2e through the C ABI from pinned host buffers. Every step copies all its inputs in
+    # (Q, K, V, the logits and the mask inputs) and its results out, three copies from and
+    # to packed buffers; the host link (~0.2 TB/s here) is the bound. Pipelined: two device
+    # buffer sets, the copies on their own stream, so that step i + 1's inputs cross the
+    # link while step i computes (a copy into a buffer waits for the step that last used
+    # it). Serial: one step at a time.
+    def packed(spec, **kw):
+        """One flat byte buffer holding the named tensors at 256-byte aligned offsets (one
+        copy moves them all), and the typed views."""
+        offs, total = [], 0
+        for name, like in spec:
+            total = (total + 255) // 256 * 256
+            nb = like.numel() * like.element_size()
+            offs.append((name, total, nb, like))
+            total += nb
+        flat = torch.empty(total, dtype=torch.uint8, **kw)
+        return flat, {n: flat[o:o + nb].view(t.dtype).view(t.shape) for n, o, nb, t in offs}
 
-    side = torch.cuda.Stream()
+    in_spec = [(k, sets[0][k]) for k in ("q", "k", "v")] + \
+              [(k, getattr(ds, k)) for k in ("state", "prev_conf", "shadow_src")]
+    lg_spec = [(k, sets[0][k]) for k in ("lx", "ls")]
+    out_names = ("conf", "token", "state_out", "counts")
+    out_spec = [(k, getattr(ds, k)) for k in out_names]
+    host_in, hv = packed(in_spec, pin_memory=True)
+    host_lg, hl = packed(lg_spec, pin_memory=True)
+    for name, t in in_spec:
+        hv[name].copy_(t)
+    for name, t in lg_spec:
+        hl[name].copy_(t)
+    h2d = host_in.numel() + host_lg.numel()
+    d2h = packed(out_spec, device="cpu")[0].numel()
+    bufs = []
+    for b in range(2):
+        d = {"o": sets[b]["o"], "w_out": torch.empty_like(ds.w_out)}
+        d["in"], views = packed(in_spec, device=dev)
+        d.update(views)
+        d["lg"], views = packed(lg_spec, device=dev)
+        d.update(views)
+        d["out"], views = packed(out_spec, device=dev)
+        d.update(views)
+        d["host_out"], d["host_views"] = packed(out_spec, pin_memory=True)
+        d["attn"] = Bd.AttentionCall(*meta, d["state"], d["prev_conf"], d["shadow_src"],
+                                     status=ds.status)
+        d["score"] = Bd.ScoreCall(ds.block_len, d["state"], wl.tau_c, wl.tau_u, wl.lam, wl.p0,
+                                  d["conf"], d["token"], d["state_out"], ds.workspace,
+                                  w_out=d["w_out"], counts=d["counts"], status=ds.status)
+        d["done"] = None
+        bufs.append(d)
+    main = torch.cuda.current_stream()
+    copy_stream = torch.cuda.Stream()
 
-    def e2e_step():
-        # Q/K/V and the mask inputs first, at the full host-link bandwidth; the logits follow
-        # on a second stream while the attention kernel runs (the link, ~0.2 TB/s here, is
-        # the bound of this measurement). Scoring waits for both.
-        main = torch.cuda.current_stream()
-        for k in ("q", "k", "v"):
-            s0[k].copy_(host_in[k], non_blocking=True)
-        for k, t in host_meta.items():
-            d_meta[k].copy_(t, non_blocking=True)
-        side.wait_event(main.record_event())
-        with torch.cuda.stream(side):
-            for k in ("lx", "ls"):
-                s0[k].copy_(host_in[k], non_blocking=True)
-        attn(s0)
-        main.wait_stream(side)
-        score(s0)
-        for k, t in outs.items():
-            host_out[k].copy_(t, non_blocking=True)
+    def e2e_step(i, nbuf):
+        b = bufs[i % nbuf]
+        with torch.cuda.stream(copy_stream):
+            if b["done"] is not None:
+                copy_stream.wait_event(b["done"])
+            b["in"].copy_(host_in, non_blocking=True)  # Q, K, V and the mask inputs
+            qkv_in = copy_stream.record_event()
+            b["lg"].copy_(host_lg, non_blocking=True)  # the logits
+            logits_in = copy_stream.record_event()
+        main.wait_event(qkv_in)
+        b["attn"](b["q"], b["k"], b["v"], b["o"])
+        main.wait_event(logits_in)
+        b["score"](b["lx"], b["ls"])
+        b["host_out"].copy_(b["out"], non_blocking=True)
+        b["done"] = main.record_event()
 
-    for _ in range(5):
-        e2e_step()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(args.e2e_steps):
-        e2e_step()
-    e1.record()
-    e1.synchronize()
-    e2e_us = e0.elapsed_time(e1) * 1e3 / args.e2e_steps
+    def e2e_run(nbuf):
+        for i in range(5):
+            e2e_step(i, nbuf)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        copy_stream.wait_stream(main)
+        for i in range(args.e2e_steps):
+            e2e_step(i, nbuf)
+        e1.record()
+        e1.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / args.e2e_steps
+
+    e2e_serial_us = e2e_run(1)
+    e2e_us = e2e_run(2)
+    e2e_ok = all(torch.equal(bufs[0]["host_views"][k], bufs[1]["host_views"][k]) and
+                 torch.equal(bufs[0]["host_views"][k], getattr(ds, k).cpu()) for k in out_names)
 
     if rank != 0:
         return
@@ -416,7 +459,8 @@ def run_ours(args, rank: int, world: int):
                     "scoring_frac_8tbs": sc_gbs / 8000.0, "scoring_bytes_per_call": sbytes},
         "clocks": clocks,
         "e2e": {"value": e2e_us, "unit": "µs", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
+                "d2h_bytes_per_step": d2h, "steps_in_flight": 2,
+                "serial_value": e2e_serial_us, "results_match_device_step": e2e_ok},
         "gpu_launches": args.steps * 3,
         "status_word": status,
     }

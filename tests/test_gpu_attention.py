@@ -66,6 +66,28 @@ def test_mask_probe_every_key(d, layout, tc):
     assert mx <= _probe_tol(wl)
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_mask_probe_last_tile_widths(d, tc):
+    """Sequences whose last 128-key tile holds 1, 15, 16, 17, 48, 63, 64, 65, 100, 127 or
+    128 keys (one tile only for the 100- and 17-row sequences): the tensor-core kernels
+    narrow that tile's products to its keys rounded up to 16, and every key must still be
+    attended exactly once (uniform attention, Q = 0)."""
+    rows = [129, 271, 144, 145, 176, 319, 192, 321, 100, 255, 256, 17]
+    specs = []
+    for i, r in enumerate(rows):
+        B = 8 if r < 64 else (16, 32)[i % 2]
+        n = r - B  # "paper" layout: one shadow row per block position
+        b0 = (n - B) if i % 3 == 0 else (n - B) // 2
+        specs.append(dict(n_orig=n, block_start=b0, block_len=B, fractions=(0.3, 0.4, 0.3)))
+    wl = W.custom(specs, 4, 2, d, probe=True, seed=61 + d)
+    assert [s.n_orig + s.n_shadow for s in wl.seqs] == rows
+    ds, o = _attend(wl)
+    mx, mean, n = P.compare_attention(wl, 0, o)
+    print("last tile widths", d, mx, mean, n)
+    assert mx <= _probe_tol(wl)
+    assert int(ds.status.item()) == 0
+
+
 def test_mask_probe_confidence_ties(tc):
     """Equal c_{t-1} among C tokens attend each other both ways (Eq. 3 uses <=)."""
     B = 48
