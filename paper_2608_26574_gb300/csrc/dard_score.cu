@@ -429,11 +429,14 @@ __device__ __forceinline__ void add_count(const ScoreParams& p, int seq, int sta
 // kExtra: the call asks for p_cur, next-step tokens or an in-place state update.
 template <class T, int VPT, bool kExtra>
 __global__ void __launch_bounds__(kScoreThreads) score_pass1(const __grid_constant__ ScoreParams p) {
-  grid_dep_launch();  // pass 2 may start loading its logits right away
   // Launched with programmatic dependent launch after whatever kernel precedes the call
   // (the LM head in a model, the attention kernel in the benchmark): this CTA may already be
-  // resident, but it touches no memory before that kernel has completed.
+  // resident, but it touches no memory before that kernel has completed. Only then may
+  // pass 2 start: it loads its logits (and the states) before it waits for pass 1, so
+  // the kernel that wrote them must have completed by the time pass 2 is launched, even
+  // when that kernel lets its own dependents start early.
   grid_dep_wait();
+  grid_dep_launch();
   using A = std::conditional_t<kExtra, AccX, Acc>;
   __shared__ A s_acc[kWarps];
   __shared__ float4 s_slots[2 * kScoreMaxSplit];
