@@ -118,29 +118,6 @@ def peaks():
     return 6800.0, 1900.0, "fallback"
 
 
-def attention_kernel(wl, sms: int = 152) -> str:
-    """The tensor-core attention kernel the library picks for this batch (the same cost
-    model as the library's launcher), or the one DARD_ATTN_TC forces."""
-    forced = os.environ.get("DARD_ATTN_TC", "")
-    if forced in ("1", "2"):
-        return f"attn_tc{forced}"
-
-    def cycles(items):
-        total = sum(n * c for n, c in items)
-        ctas = sum(n for n, _ in items)
-        longest = max([c for n, c in items if n > 0] or [0.0])
-        return longest if ctas <= sms else total / sms + 0.5 * longest
-
-    one, two = [], []
-    for s in wl.seqs:
-        kt = (s.rows + 127) // 128
-        tiles = (s.rows - s.query_start + 127) // 128
-        one.append((tiles * wl.hq, 14700.0 + 1480.0 * kt))
-        two.append(((tiles // 2) * wl.hq, 13900.0 + 3770.0 * kt))
-        two.append(((tiles % 2) * wl.hq, 8800.0 + 3000.0 * kt))
-    return "attn_tc2" if cycles(two) < cycles(one) else "attn_tc1"
-
-
 def traffic_for(kernel: str, source: str, per_launch_units: float):
     """DRAM bytes per launch from profiles/traffic.txt, if recorded for this source hash."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
@@ -435,7 +412,9 @@ def run_ours(args, rank: int, world: int):
     if rank != 0:
         return
     hbm, bf16, peak_kind = peaks()
-    attn_kernel = attention_kernel(wl)
+    # the kernel the library launches for this batch (its own cost model, or DARD_ATTN_TC)
+    attn_kernel = {1: "attn_tc1", 2: "attn_tc2", 3: "attn_simt"}[
+        ds.attention_call().kernel(q0, k0, v0, sets[0]["o"])]
     flops = W.attention_flops(wl)
     sbytes = W.scoring_bytes(wl)
     att_tflops = flops / (attn_us * 1e-6) / 1e12

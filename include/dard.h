@@ -142,6 +142,16 @@ typedef struct {
  * _ALIGN, _CUDA. */
 dard_status dard_step_attention(const dard_attn_args* args, void* stream /* cudaStream_t */);
 
+/* The attention kernel dard_step_attention would launch for these arguments, without
+ * launching anything: *kernel = 1 or 2 (the tensor-core kernel with one or two 128-row
+ * query tiles per CTA, as the cost model or DARD_ATTN_TC picks), 3 (the fp32 CUDA-core
+ * kernel), or 0 (no query rows, no launch). The arguments go through the same host
+ * validation as dard_step_attention and fail with the same codes; device pointers are
+ * checked but never read. The cost model uses the current device's SM count (148 when no
+ * device is visible, so that the choice can be planned on a host without one). An
+ * interface addition: the paper has no counterpart. */
+dard_status dard_attention_kernel(const dard_attn_args* args, int32_t* kernel);
+
 /* ------------------------------------------------------------------------------------- *
  * Confidence scoring and state transition (Eq. 1, Eq. 5-8, Algorithm 1).
  *

@@ -64,6 +64,8 @@ _lib = None
 # Exported entry points: name -> (restype, argtypes)
 EXPORTS = {
     "dard_step_attention": (ctypes.c_int, [ctypes.POINTER(AttnArgs), ctypes.c_void_p]),
+    "dard_attention_kernel": (ctypes.c_int, [ctypes.POINTER(AttnArgs),
+                                             ctypes.POINTER(ctypes.c_int32)]),
     "dard_score_and_transition": (ctypes.c_int, [ctypes.POINTER(ScoreArgs), ctypes.c_void_p]),
     "dard_score_and_transition_noalloc": (ctypes.c_int, [ctypes.POINTER(ScoreArgs),
                                                          ctypes.c_void_p]),
@@ -208,6 +210,21 @@ class AttentionCall:
 
     def __call__(self, q, k, v, o, stream=None):
         """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d]."""
+        dev = self._bind(q, k, v, o)
+        _check(self._fn(self._ref, _stream_handle(stream, dev)), "dard_step_attention")
+
+    def kernel(self, q, k, v, o) -> int:
+        """The kernel a call on these tensors launches, without launching it: 1 or 2 (the
+        tensor-core kernel with one or two query tiles per CTA), 3 (fp32 CUDA cores), 0 (no
+        query rows)."""
+        self._bind(q, k, v, o)
+        out = ctypes.c_int32(-1)
+        _check(lib().dard_attention_kernel(self._ref, ctypes.byref(out)), "dard_attention_kernel")
+        return int(out.value)
+
+    def _bind(self, q, k, v, o) -> int:
+        """Checks q, k, v and o against the metadata and sets their pointers; returns the
+        device index."""
         if not (q.is_cuda and k.is_cuda and v.is_cuda and o.is_cuda):
             raise ValueError("q, k, v and o must be device tensors")
         if not (q.is_contiguous() and k.is_contiguous() and v.is_contiguous()
@@ -230,7 +247,7 @@ class AttentionCall:
         a.q, a.k, a.v, a.o = q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr()
         a.dtype = _dtype_code(q)
         a.hq, a.hkv, a.head_dim = qs[1], ks[1], qs[2]
-        _check(self._fn(self._ref, _stream_handle(stream, dev)), "dard_step_attention")
+        return dev
 
 
 def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, state,
@@ -240,6 +257,14 @@ def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, 
     ``query_start`` (per sequence, optional): first query row; earlier rows are keys only."""
     AttentionCall(n_orig, block_start, block_len, shadow_len, state, prev_conf, shadow_src,
                   scale=scale, status=status, query_start=query_start)(q, k, v, o, stream)
+
+
+def dard_attention_kernel(q, k, v, o, n_orig, block_start, block_len, shadow_len, state,
+                          prev_conf, shadow_src, scale: float = 0.0, query_start=None) -> int:
+    """The kernel dard_step_attention would launch for these arguments (see
+    ``AttentionCall.kernel``), without launching anything."""
+    return AttentionCall(n_orig, block_start, block_len, shadow_len, state, prev_conf,
+                         shadow_src, scale=scale, query_start=query_start).kernel(q, k, v, o)
 
 
 def dard_score_workspace_size(rows: int, vocab: int, num_seqs: int) -> int:

@@ -54,9 +54,14 @@ const char* dard_last_error(void) { return g_err; }
 
 int32_t dard_version(void) { return 100; }
 
-dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Host-side validation of an attention call and its launch plan (the per-sequence
+// descriptors, the longest-first work order and the kernel parameters). Touches no device.
+dard_status prepare_attention(const dard_attn_args* a, dard::AttnParams& p) {
   using namespace dard;
-  g_err[0] = '\0';
   if (!a) return fail(DARD_ERR_NULL, "args is NULL");
   if (!a->q || !a->k || !a->v || !a->o) return fail(DARD_ERR_NULL, "q, k, v or o is NULL");
   if (!a->n_orig || !a->block_start || !a->block_len || !a->shadow_len)
@@ -74,7 +79,6 @@ dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
   if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o))
     return fail(DARD_ERR_ALIGN, "q, k, v and o must be 16-byte aligned");
 
-  AttnParams p;
   memset(&p, 0, sizeof(p));
   long long rows = 0, blk = 0, sh = 0;
   std::vector<long long> cost(a->num_seqs);
@@ -143,8 +147,32 @@ dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
   p.num_seqs = a->num_seqs;
   p.scale = a->scale > 0.f ? a->scale : 1.0f / std::sqrt(static_cast<float>(a->head_dim));
   p.scale_log2 = p.scale * 1.4426950408889634f;
+  return DARD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
+  using namespace dard;
+  g_err[0] = '\0';
+  AttnParams p;
+  const dard_status st = prepare_attention(a, p);
+  if (st != DARD_OK) return st;
   if (p.total_work == 0) return DARD_OK;  // no query rows (every query_start at the end)
   return launch_attention(*a, p, static_cast<cudaStream_t>(stream), g_err, sizeof(g_err));
+}
+
+dard_status dard_attention_kernel(const dard_attn_args* a, int32_t* kernel) {
+  using namespace dard;
+  g_err[0] = '\0';
+  if (!kernel) return fail(DARD_ERR_NULL, "kernel is NULL");
+  AttnParams p;
+  const dard_status st = prepare_attention(a, p);
+  if (st != DARD_OK) return st;
+  *kernel = p.total_work == 0 ? 0 : attention_kernel_choice(*a, p);
+  return DARD_OK;
 }
 
 size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs) {

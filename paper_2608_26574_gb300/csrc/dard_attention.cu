@@ -1285,16 +1285,13 @@ int sm_count() {
 }
 
 template <int D>
-cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
+cudaError_t launch_tc(const AttnParams& p, int kernel, cudaStream_t stream) {
   static std::atomic<uint64_t> attr1_done{0}, attr2_done{0};
   CUtensorMap mq, mk, mv;
   if (!make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
       !make_map(&mv, p.v, p.hkv, D, p.total_rows, kTN))
     return cudaErrorInvalidValue;
-  // DARD_ATTN_TC=1 or 2 forces one kernel (tests and tuning); anything else: the model
-  const char* force = std::getenv("DARD_ATTN_TC");
-  const int forced = force ? std::atoi(force) : 0;
-  if (forced == 2 || (forced != 1 && prefer_tc2(p, sm_count()))) {
+  if (kernel == 2) {
     if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM)) return cudaErrorInvalidValue;
     const size_t smem = tc2_smem_bytes<D>();
     cudaError_t e = ensure_smem_attr(attn_tc2<D>, smem, attr2_done);
@@ -1311,15 +1308,25 @@ cudaError_t launch_tc(const AttnParams& p, cudaStream_t stream) {
 
 }  // namespace
 
+int attention_kernel_choice(const dard_attn_args& a, const AttnParams& p) {
+  if (a.dtype == DARD_F32) return 3;
+  // DARD_ATTN_TC=1 or 2 forces one kernel (tests and tuning); anything else: the model
+  const char* force = std::getenv("DARD_ATTN_TC");
+  const int forced = force ? std::atoi(force) : 0;
+  if (forced == 1 || forced == 2) return forced;
+  return prefer_tc2(p, sm_count()) ? 2 : 1;
+}
+
 dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
                              char* err, size_t err_len) {
   cudaError_t e;
-  if (a.dtype == DARD_F32) {
+  const int kernel = attention_kernel_choice(a, p);
+  if (kernel == 3) {
     if (a.head_dim == 64) attn_simt<64><<<p.total_work, 128, 0, stream>>>(p);
     else attn_simt<128><<<p.total_work, 128, 0, stream>>>(p);
     e = cudaGetLastError();
   } else {
-    e = a.head_dim == 64 ? launch_tc<64>(p, stream) : launch_tc<128>(p, stream);
+    e = a.head_dim == 64 ? launch_tc<64>(p, kernel, stream) : launch_tc<128>(p, kernel, stream);
   }
   if (e != cudaSuccess) {
     snprintf(err, err_len, "attention launch failed: %s", cudaGetErrorString(e));

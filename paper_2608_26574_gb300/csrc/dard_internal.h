@@ -47,6 +47,11 @@ struct AttnParams {
   SeqDesc seq[DARD_MAX_SEQS];
 };
 
+// The kernel a validated call launches: 1 or 2 (the tensor-core kernel with one or two
+// query tiles per CTA), 3 (the fp32 CUDA-core kernel). Shared by the launcher and by
+// dard_attention_kernel(); reads DARD_ATTN_TC and the current device's SM count.
+int attention_kernel_choice(const dard_attn_args& a, const AttnParams& p);
+
 dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
                              char* err, size_t err_len);
 

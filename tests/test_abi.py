@@ -91,6 +91,54 @@ def test_attention_null_args(lib):
     assert lib.dard_step_attention(None, None) == 1
 
 
+@pytest.mark.parametrize("change,code", [
+    ({"q": None}, 1), ({"dtype": 7}, 3), ({"num_seqs": 0}, 2), ({"hq": 6, "hkv": 4}, 2),
+    ({"head_dim": 96}, 4), ({"scale": -1.0}, 3), ({"q": 0x10008}, 6),
+    ({"bl": np.array([129], np.int32)}, 2), ({"qs": np.array([97], np.int32)}, 2),
+])
+def test_attention_kernel_query_validates_like_the_launch(lib, change, code):
+    """dard_attention_kernel runs the launch's host validation and returns its codes,
+    leaving the output untouched."""
+    a, keep = _attn_args(**change)
+    out = ctypes.c_int32(-1)
+    assert lib.dard_attention_kernel(ctypes.byref(a), ctypes.byref(out)) == code
+    assert out.value == -1
+
+
+def test_attention_kernel_query_null(lib):
+    a, keep = _attn_args()
+    assert lib.dard_attention_kernel(ctypes.byref(a), None) == 1
+    assert lib.dard_attention_kernel(None, ctypes.byref(ctypes.c_int32())) == 1
+
+
+def _kernel(lib, **kw):
+    a, keep = _attn_args(**kw)
+    out = ctypes.c_int32(-1)
+    assert lib.dard_attention_kernel(ctypes.byref(a), ctypes.byref(out)) == 0
+    return out.value
+
+
+def test_attention_kernel_choice(lib, monkeypatch):
+    """The launcher's choice, planned on the host (nothing is launched; the device pointers
+    are never read). Cases whose answer holds at 148 or 152 SMs: the 8B layer (one wave of
+    query-tile pairs) takes the two-tile kernel, a 5184-row GQA sequence (about eight waves
+    of single tiles) the one-tile kernel, fp32 the CUDA-core kernel, and a batch without
+    query rows no kernel; DARD_ATTN_TC forces either tensor-core kernel."""
+    monkeypatch.delenv("DARD_ATTN_TC", raising=False)
+    i32 = lambda *x: np.array(x, np.int32)  # noqa: E731
+    layer_8b = dict(n=i32(768), b0=i32(608), bl=i32(32), sl=i32(32), hq=32, hkv=32,
+                    head_dim=128)
+    gqa = dict(n=i32(5120), b0=i32(4608), bl=i32(64), sl=i32(64), hq=28, hkv=4, head_dim=128)
+    assert _kernel(lib, **layer_8b) == 2
+    assert _kernel(lib, **gqa) == 1
+    assert _kernel(lib, **layer_8b, dtype=B.DARD_F32) == 3
+    assert _kernel(lib, **layer_8b, qs=i32(800)) == 0
+    monkeypatch.setenv("DARD_ATTN_TC", "1")
+    assert _kernel(lib, **layer_8b) == 1
+    monkeypatch.setenv("DARD_ATTN_TC", "2")
+    assert _kernel(lib, **gqa) == 2
+
+
 def _score_args(**kw):
     bl = kw.pop("bl", np.array([32], np.int32))
     a = B.ScoreArgs()

@@ -154,3 +154,23 @@ def test_score_call_rejects_mismatched_tensors():
             (a if key in a else extra)[key] = val
         with pytest.raises(ValueError):
             B.ScoreCall(*args, a["conf"], a["token"], a["state_out"], ds.workspace, **extra)
+
+
+@pytest.mark.gpu
+def test_attention_kernel_query(monkeypatch):
+    """The kernel the launcher picks, asked without launching: the two-tile kernel for the
+    8B layer, the one-tile kernel for a long GQA sequence, the CUDA-core kernel for fp32,
+    and what DARD_ATTN_TC forces."""
+    monkeypatch.delenv("DARD_ATTN_TC", raising=False)
+    for name, want in (("8b", 2), ("gqa", 1), ("tiny", 3)):
+        wl = W.make(name, scoring=False, layers=1)
+        ds = DeviceStep(wl, layers=[0], scoring=False)
+        q, k, v, o = ds.layers[0]
+        assert ds.attention_call().kernel(q, k, v, o) == want, name
+        assert B.dard_attention_kernel(q, k, v, o, ds.n_orig, ds.block_start, ds.block_len,
+                                       ds.shadow_len, ds.state, ds.prev_conf,
+                                       ds.shadow_src) == want
+        if want != 3:
+            monkeypatch.setenv("DARD_ATTN_TC", str(3 - want))
+            assert ds.attention_call().kernel(q, k, v, o) == 3 - want
+            monkeypatch.delenv("DARD_ATTN_TC")
