@@ -1140,55 +1140,85 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
 }
 
 // ---------------------------------------------------------------- fp32 CUDA-core path
+// Two threads per query row (a CTA holds a 128-row query tile of one head): each owns the
+// row's even or odd elements of q and of the O accumulator in registers. The sequence's
+// keys pass through shared memory 32 rows at a time (K and V, read as broadcasts: the two
+// threads of a row read neighbouring words); per visible key the pair adds up its partial
+// dot products with one shuffle and updates its own online softmax. Masking as on the
+// tensor-core path, by key_visible().
 template <int D>
-__global__ void __launch_bounds__(128) attn_simt(const __grid_constant__ AttnParams p) {
-  constexpr int kPer = D / 32;
+__global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnParams p) {
+  constexpr int kH = D / 2;  // elements per thread
+  constexpr int kKT = 32;    // keys per shared-memory tile
   __shared__ BlockInfo bi;
+  __shared__ float sK[kKT][D], sV[kKT][D];
   int seq, qt, h;
   decode_work(p, blockIdx.x, seq, qt, h);
   const SeqDesc sd = p.seq[seq];
   const int rows_seq = sd.n_orig + sd.slen;
   const int g = h / (p.hq / p.hkv);
-  load_block_info(p, sd, bi, qt == 0 && h == 0);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x < 128) load_block_info(p, sd, bi, qt == 0 && h == 0);  // warps 0-3
+  __syncthreads();
+  const int t = threadIdx.x >> 1, half = threadIdx.x & 1;
+  const unsigned pair = 3u << ((threadIdx.x & 31) & ~1);  // this thread and its partner
+  const int r = sd.q_start + qt * kBM + t;  // sequence-relative query row
+  const bool active = r < rows_seq;
+  RowInfo q{0, kStateU, 0.f, -1, 0};
+  if (active) q = row_info(sd, bi, r);
+  const bool live = active && q.store;
   const float* Q = static_cast<const float*>(p.q);
   const float* K = static_cast<const float*>(p.k);
   const float* V = static_cast<const float*>(p.v);
   float* O = static_cast<float*>(p.o);
-  const float scale = p.scale;
-  for (int rr = 0; rr < 32; ++rr) {
-    const int r = sd.q_start + qt * kBM + warp * 32 + rr;
-    if (r >= rows_seq) break;
-    const RowInfo q = row_info(sd, bi, r);
-    if (!q.store) continue;
-    const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D;
-    float qv[kPer], acc[kPer];
+  const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D + half;
+  float qv[kH], acc[kH];
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) {
-      qv[e] = Q[qoff + lane + 32 * e];
-      acc[e] = 0.f;
+  for (int e = 0; e < kH; ++e) {
+    qv[e] = live ? Q[qoff + 2 * e] : 0.f;
+    acc[e] = 0.f;
+  }
+  float m = -INFINITY, l = 0.f;
+  for (int kt0 = 0; kt0 < rows_seq; kt0 += kKT) {
+    __syncthreads();  // the previous tile has been read
+    for (int idx = threadIdx.x; idx < kKT * D; idx += 256) {
+      const int kk = idx / D, d = idx % D;
+      const int kr = kt0 + kk;
+      float kx = 0.f, vx = 0.f;
+      if (kr < rows_seq) {
+        const size_t off = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D + d;
+        kx = K[off];
+        vx = V[off];
+      }
+      sK[kk][d] = kx;
+      sV[kk][d] = vx;
     }
-    float m = -INFINITY, l = 0.f;
-    for (int kr = 0; kr < rows_seq; ++kr) {
-      if (!key_visible(q, bi, sd, kr)) continue;
-      const size_t koff = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D;
+    __syncthreads();
+    if (!live) continue;
+    const int nk = min(kKT, rows_seq - kt0);
+    for (int kk = 0; kk < nk; ++kk) {
+      if (!key_visible(q, bi, sd, kt0 + kk)) continue;  // the same for both threads of a row
       float dot = 0.f;
 #pragma unroll
-      for (int e = 0; e < kPer; ++e) dot = fmaf(qv[e], K[koff + lane + 32 * e], dot);
+      for (int e = 0; e < kH; ++e) dot = fmaf(qv[e], sK[kk][2 * e + half], dot);
+      dot += __shfl_xor_sync(pair, dot, 1);
+      const float z = dot * p.scale;
+      if (z > m) {
+        const float alpha = (m == -INFINITY) ? 0.f : expf(m - z);
+        l *= alpha;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-      const float z = dot * scale;
-      const float m_new = fmaxf(m, z);
-      const float alpha = (m == -INFINITY) ? 0.f : expf(m - m_new);
-      const float pz = expf(z - m_new);
-      l = l * alpha + pz;
+        for (int e = 0; e < kH; ++e) acc[e] *= alpha;
+        m = z;
+      }
+      const float pz = expf(z - m);
+      l += pz;
 #pragma unroll
-      for (int e = 0; e < kPer; ++e) acc[e] = fmaf(pz, V[koff + lane + 32 * e], acc[e] * alpha);
-      m = m_new;
+      for (int e = 0; e < kH; ++e) acc[e] = fmaf(pz, sV[kk][2 * e + half], acc[e]);
     }
+  }
+  if (live) {
     const float inv_l = 1.0f / l;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) O[qoff + lane + 32 * e] = acc[e] * inv_l;
+    for (int e = 0; e < kH; ++e) O[qoff + 2 * e] = acc[e] * inv_l;
   }
 }
 
@@ -1322,8 +1352,8 @@ dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_
   cudaError_t e;
   const int kernel = attention_kernel_choice(a, p);
   if (kernel == 3) {
-    if (a.head_dim == 64) attn_simt<64><<<p.total_work, 128, 0, stream>>>(p);
-    else attn_simt<128><<<p.total_work, 128, 0, stream>>>(p);
+    if (a.head_dim == 64) attn_simt<64><<<p.total_work, 256, 0, stream>>>(p);
+    else attn_simt<128><<<p.total_work, 256, 0, stream>>>(p);
     e = cudaGetLastError();
   } else {
     e = a.head_dim == 64 ? launch_tc<64>(p, kernel, stream) : launch_tc<128>(p, kernel, stream);

@@ -108,6 +108,26 @@ def test_attention_run_to_run_identical(tc):
     assert int(ds.status.item()) == 0
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_attention_fp32(d):
+    """The fp32 CUDA-core kernel at both head dims: every key selection (uniform attention,
+    Q = 0) and random values against the oracle, over two sequences with blocks, shadow rows
+    in both layouts and grouped heads. fp32 throughout: the error stays near fp32 rounding."""
+    specs = [dict(n_orig=150, block_start=60, block_len=40, fractions=(0.3, 0.4, 0.3)),
+             dict(n_orig=70, block_start=0, block_len=33, fractions=(0.4, 0.3, 0.3),
+                  shadow="candidates")]
+    wl = W.custom(specs, 4, 2, d, dtype="f32", probe=True, seed=71 + d)
+    _, o = _attend(wl)
+    mx, _, _ = P.compare_attention(wl, 0, o)
+    assert mx <= _probe_tol(wl)
+    wl = W.custom(specs, 4, 2, d, dtype="f32", seed=81 + d, qkv_std=1.0)
+    ds, o = _attend(wl)
+    mx, mean, n = P.compare_attention(wl, 0, o)
+    print("fp32", d, mx, mean, n)
+    assert mx <= 2e-4
+    assert int(ds.status.item()) == 0
+
+
 def test_mask_probe_confidence_ties(tc):
     """Equal c_{t-1} among C tokens attend each other both ways (Eq. 3 uses <=)."""
     B = 48
