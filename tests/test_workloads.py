@@ -44,3 +44,25 @@ def test_seeded_reproducible():
     b = W.make("tiny")
     assert (a.q[0] == b.q[0]).all() and (a.logits_s == b.logits_s).all()
     assert (a.seqs[0].state == b.seqs[0].state).all()
+
+
+def test_algorithmic_work_closed_forms():
+    """The roofline numerators, from each configuration's definition by hand: attention
+    4·d·(rows − query_start)·N·Hq FLOPs, scoring V·esize·(B + |M|) bytes."""
+    from paper_2608_26574_gb300 import workloads as W
+    wl = W.make("8b", attention=False, scoring=False)
+    assert W.attention_flops(wl) == 4 * 128 * 800 * 768 * 32 == 10_066_329_600
+    wl = W.make("8b", layout="candidates", attention=False, scoring=False)
+    assert W.attention_flops(wl) == 4 * 128 * (768 + 8) * 768 * 32  # 8 C positions
+    wl = W.make("8b", prefix=True, attention=False, scoring=False)
+    assert W.attention_flops(wl) == 4 * 128 * (800 - 512) * 768 * 32  # queries after the prompt
+    wl = W.make("gqa", attention=False, scoring=False)
+    assert W.attention_flops(wl) == 4 * 128 * 5184 * 5120 * 28 == 380_507_258_880
+    wl = W.make("tiny", attention=False, scoring=False)
+    assert W.attention_flops(wl) == 4 * 64 * 96 * 64 * 4
+    wl = W.make("8b", attention=False)
+    assert W.scoring_bytes(wl) == 126464 * 2 * (32 + 16) == 12_140_544  # 16 M rows, bf16
+    wl = W.make("gqa", attention=False)
+    assert W.scoring_bytes(wl) == 152064 * 2 * (64 + 19)  # 19 M rows
+    wl = W.make("tiny", attention=False)
+    assert W.scoring_bytes(wl) == 1024 * 4 * (32 + 13)  # fp32 logits, 13 M rows
