@@ -19,7 +19,7 @@ and are therefore formed in float32 exactly as the kernel forms them:
 ``mix = ls + w * (lx - ls)`` with each operation rounded to float32 (the paper's
 ``w*lx + (1-w)*ls`` regrouped; see ``mix_logits``).
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open (the readings below):
   R1  keys of M positions seen by C queries and by M shadow queries come from s;
   R2  a shadow query s^i always sees its own shadow key s^i (no self leak), an original
       query x^i always sees x^i;

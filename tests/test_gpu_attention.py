@@ -38,7 +38,7 @@ def test_attention_configs(name, layout, sample, tc):
         ds, o = _attend(wl, li)
         mx, mean, n = P.compare_attention(wl, li, o, sample=sample)
         print(name, layout, li, "max", mx, "mean", mean, "rows", n)
-        assert mx <= P.att_tol(wl, li) and mean <= P.ATT_MEAN_ABS
+        assert mx <= P.ATT_MAX_ABS and mean <= P.ATT_MEAN_ABS
         assert int(ds.status.item()) == 0
 
 
@@ -215,7 +215,8 @@ def test_attention_prefix_cached(name, sample, tc):
     torch.cuda.synchronize()
     o = out.float().cpu().numpy()
     mx, mean, n = P.compare_attention(wl, 0, o, sample=sample)
-    assert mx <= P.att_tol(wl, 0) and mean <= P.ATT_MEAN_ABS
+    print(name, "prefix", "max", mx, "mean", mean, "rows", n)
+    assert mx <= P.ATT_MAX_ABS and mean <= P.ATT_MEAN_ABS
     offs = wl.row_offsets()
     for si, s in enumerate(wl.seqs):
         assert s.query_start == s.prompt > 0

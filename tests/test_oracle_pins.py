@@ -568,3 +568,68 @@ def test_order_keys_reproduce_the_ablation_orderings():
     assert orc.order_key(orc.ORDER_CONFIDENCE, 0.7, 2.0, 0.1, 3) == 0.7
     assert orc.order_key(orc.ORDER_ENTROPY, 0.7, 2.0, 0.1, 3) == -2.0
     assert orc.order_key(orc.ORDER_MARGIN, 0.7, 2.0, 0.1, 3) == 0.1
+
+
+# ---------------------------------------------------------------- near-tie gap, reading R7
+def test_top2_gap_closed_forms():
+    """The near-tie exclusion of the parity checks (reading R5: argmax ties go to the lowest
+    index, so a gap under rounding may flip it): the gap is the largest entry minus the
+    second largest, a repeated maximum gives 0, a single entry gives inf."""
+    assert orc.top2_gap(np.array([1.0, 5.0, 3.0], np.float32)) == 2.0
+    assert orc.top2_gap(np.array([-4.0, -1.5, -9.0, -2.0], np.float32)) == 0.5
+    assert orc.top2_gap(np.array([3.0, 7.0, 7.0], np.float32)) == 0.0
+    assert orc.top2_gap(np.array([7.0, 1.0, 7.0, 7.0], np.float32)) == 0.0
+    assert orc.top2_gap(np.array([2.5], np.float32)) == math.inf
+    assert orc.top2_gap(np.array([-np.inf, 2.0], np.float32)) == math.inf
+    # the gap is never negative, whatever the order of the entries
+    assert orc.top2_gap(np.array([9.0, 8.0, 1.0], np.float32)) == 1.0
+
+
+def test_top2_gap_brute_force():
+    """Against the definition over all pairs: max over i != j of x_i - x_j restricted to
+    i = an argmax, i.e. the maximum minus the largest entry at any other index."""
+    rng = np.random.default_rng(41)
+    for _ in range(200):
+        V = int(rng.integers(2, 9))
+        x = rng.integers(-3, 4, size=V).astype(np.float32) * np.float32(0.25)
+        a = int(np.argmax(x))
+        others = [float(x[j]) for j in range(V) if j != a]
+        assert orc.top2_gap(x) == float(x[a]) - max(others)
+
+
+@pytest.mark.parametrize("bad", [3, 7, 255])
+def test_state_byte_above_two_is_masked(bad):
+    """Reading R7: a state byte above 2 behaves exactly as M, in the mask (every query's
+    attended set, Sec. 3.2) and in scoring (Algorithm 1: the row is mixed and decided as an
+    M row and counted as M)."""
+    rng = np.random.default_rng(43 + bad)
+    for shadow in ("paper", "candidates"):
+        lay = _rand_layout(rng, B=10, shadow=shadow)
+        st = lay.state.copy()
+        m_rows = np.flatnonzero(st == M)
+        if len(m_rows) == 0:
+            st[0] = M
+            m_rows = np.array([0])
+        ref = SeqLayout(lay.n_orig, lay.block_start, st, lay.prev_conf,
+                        np.asarray(lay.shadow_src, np.int32) if shadow == "paper"
+                        else lay.block_start + np.flatnonzero(st == C).astype(np.int32))
+        bad_st = st.copy()
+        bad_st[m_rows] = bad
+        odd = SeqLayout(ref.n_orig, ref.block_start, bad_st, ref.prev_conf, ref.shadow_src)
+        assert np.array_equal(orc.attention_mask(odd), orc.attention_mask(ref))
+    V = 96
+    state = np.array([M, C, U, M, C, M], np.uint8)
+    lx = rng.standard_normal((6, V)).astype(np.float32)
+    ls = rng.standard_normal((6, V)).astype(np.float32)
+    ls[1, 5] += 9.0   # promoted C row
+    ls[4, 7] -= 0.0   # C row that stays low (demoted)
+    want = orc.score_block(lx, ls, state, 0.4, 0.9)
+    odd_state = state.copy()
+    odd_state[[0, 5]] = bad
+    got = orc.score_block(lx, ls, odd_state, 0.4, 0.9)
+    assert np.array_equal(got.state_out, want.state_out)
+    assert np.array_equal(got.token, want.token)
+    assert np.array_equal(got.conf, want.conf)
+    assert np.array_equal(got.w, want.w, equal_nan=True)
+    assert list(got.counts) == list(want.counts)
+    assert got.promoted == want.promoted and got.demoted == want.demoted
