@@ -413,7 +413,7 @@ def run_ours(args, rank: int, world: int):
         return
     hbm, bf16, peak_kind = peaks()
     # the kernel the library launches for this batch (its own cost model, or DARD_ATTN_TC)
-    attn_kernel = {1: "attn_tc1", 2: "attn_tc2", 3: "attn_simt"}[
+    attn_kernel = {1: "attn_tc1", 2: "attn_tc2", 3: "attn_simt", 4: "attn_pair"}[
         ds.attention_call().kernel(q0, k0, v0, sets[0]["o"])]
     flops = W.attention_flops(wl)
     sbytes = W.scoring_bytes(wl)

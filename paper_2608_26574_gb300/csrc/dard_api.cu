@@ -147,6 +147,8 @@ dard_status prepare_attention(const dard_attn_args* a, dard::AttnParams& p) {
   p.num_seqs = a->num_seqs;
   p.scale = a->scale > 0.f ? a->scale : 1.0f / std::sqrt(static_cast<float>(a->head_dim));
   p.scale_log2 = p.scale * 1.4426950408889634f;
+  p.wait_cycles = 0;
+  p.test_drop_kv = -1;
   return DARD_OK;
 }
 

@@ -35,6 +35,9 @@ struct AttnParams {
   uint32_t* status;
   float scale;               // softmax scale
   float scale_log2;          // scale * log2(e)
+  long long wait_cycles;     // bound of every in-kernel wait in SM cycles (0: the default)
+  int32_t test_drop_kv;      // test hook: the K/V stage use whose K copy is never issued
+                             // (a wait then runs out); -1 in normal operation
   int32_t hq, hkv, head_dim, num_seqs;
   int32_t total_rows;
   int32_t total_work;        // number of (sequence, q-tile, head) work items
@@ -51,6 +54,11 @@ struct AttnParams {
 // query tiles per CTA), 3 (the fp32 CUDA-core kernel). Shared by the launcher and by
 // dard_attention_kernel(); reads DARD_ATTN_TC and the current device's SM count.
 int attention_kernel_choice(const dard_attn_args& a, const AttnParams& p);
+
+// The pair kernel (two CTAs per 256-row work item, tcgen05 cta_group::2, head_dim 128,
+// persistent over work items): launch, and the number of clusters a launch uses.
+cudaError_t launch_pair_attention(const AttnParams& p, cudaStream_t stream);
+int pair_clusters_for(const AttnParams& p);
 
 dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
                              char* err, size_t err_len);

@@ -11,9 +11,10 @@ from . import parity as P
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(params=["1", "2"])
+@pytest.fixture(params=["1", "2", "4"])
 def tc(request, monkeypatch):
-    """Runs the test once per tensor-core kernel (one or two query tiles per CTA)."""
+    """Runs the test once per tensor-core kernel: one or two query tiles per CTA (1, 2), and
+    the CTA-pair kernel (4, head_dim 128; head_dim 64 falls back to the model's choice)."""
     monkeypatch.setenv("DARD_ATTN_TC", request.param)
     return request.param
 
