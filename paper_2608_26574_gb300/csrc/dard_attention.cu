@@ -23,14 +23,14 @@
 //   bandwidth goes to K and V only.
 //
 // attn_tc2: two 128-row query tiles of the same (sequence, head), so that every K/V tile
-// serves 256 rows; 10 warps:
+// serves 256 rows; 11 warps:
 //   warps 4q .. 4q + 3  softmax and epilogue of tile q, one thread per query row;
 //   warp 8              TMA producer: both Q tiles, then K and V through 2 stages each;
-//   warp 9              TMEM allocator and MMA issuer, in the order S_0(0) S_1(0) |
-//                       PV_0(j) S_0(j+1) PV_1(j) S_1(j+1) | ... (Q from shared memory).
+//   warp 9              TMEM allocator and S issuer: S_q(j) = Q_q K(j)^T (Q from shared
+//                       memory), once PV_q(j - 1) has read P_q(j - 1) out of S_q's columns;
+//   warp 10             PV issuer: O_q += P_q(j) V(j) once P_q(j) is stored.
 //   TMEM: S_0, S_1 [0, 256) with P_q(j) written over the first 64 columns of S_q(j),
-//   O_0, O_1 [256, 256 + 2D). S_q(j+1) is issued once PV_q(j) has read P_q(j).
-//
+//   O_0, O_1 [256, 256 + 2D).
 // Both keep a per-row running maximum and rescale O in TMEM only when the maximum grows by
 // more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
 // fp32 path (attn_simt): CUDA-core kernel, one warp per query row, same mask logic.
@@ -46,13 +46,14 @@ namespace dard {
 namespace {
 
 constexpr int kTc1Threads = 352;  // attn_tc1: 8 softmax warps, producer, PV issuer, S issuer
-constexpr int kTc2Threads = 320;  // attn_tc2: 2 x 4 softmax warps, TMA producer, MMA issuer
+constexpr int kTc2Threads = 352;  // attn_tc2: 2 x 4 softmax warps, TMA producer, S and PV issuers
 
 constexpr int kQT = 2;   // query tiles per CTA (the same sequence and head)
 constexpr int kNK = 2;   // TMA stages for K
 constexpr int kNV = 2;   // TMA stages for V
 constexpr int kWProd = 2 * kQT * 2;  // warp 8: TMA producer
-constexpr int kWMma = kWProd + 1;    // warp 9: TMEM allocator and MMA issuer
+constexpr int kWMma = kWProd + 1;    // warp 9: TMEM allocator and S issuer
+constexpr int kWPv = kWProd + 2;     // warp 10: PV issuer
 
 // Named barriers: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = the 8 softmax warps,
 // then per kernel: attn_tc1 3 + q = the two warps sharing TMEM lane quarter q; attn_tc2
@@ -663,58 +664,57 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       }
     }
   } else if (warp == kWMma) {
-    // ------------------------------------------------------------ MMA issuer
-    // Tensor-pipe order: S_0(0) S_1(0) | PV_0(j) S_0(j+1) PV_1(j) S_1(j+1) | ... The softmax
-    // of tile 0 runs while the pipe does PV_1 and S_1, and the other way round. S_q(j+1)
-    // overwrites the P_q(j) that PV_q(j) reads, so it is issued once PV_q(j) has completed.
+    // ------------------------------------------------------------ S issuer
+    // S_q(j) = Q_q K(j)^T once K(j) has landed and, for j > 0, PV_q(j - 1) has completed
+    // (S_q(j) overwrites the P_q(j - 1) that PV_q(j - 1) reads). The PV products come from
+    // a second issuer thread: one thread issuing both kinds of product in turn leaves the
+    // tensor pipe at about two thirds of its rate on this GPU.
     if (lane == 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
-      constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
-      const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK), av = smem_u32(sV);
-      auto issue_s = [&](int q, int j) {
-        const uint32_t qaddr = aq + q * kTileBytes, kaddr = ak + (j % kNK) * kTileBytes;
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t off = (ks >> 2) * kKSub + (ks & 3) * 32;
-          mma_ss(tS0 + q * kTN, smem_desc_sw128(qaddr + off, 16, 1024),
-                 smem_desc_sw128(kaddr + off, 16, 1024), kIdS, ks > 0);
-        }
-        mma_commit(&ctl.s_full[q]);
-      };
-      auto issue_pv = [&](int q, int j) {
-        const uint32_t vaddr = av + (j % kNV) * kTileBytes;
-#pragma unroll
-        for (int ks = 0; ks < kTN / 16; ++ks)
-          mma_ts(tO0 + q * D, tS0 + q * kTN + ks * 8,
-                 smem_desc_sw128(vaddr + ks * 2048, kKSub, 1024), kIdO,
-                 (j > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&ctl.pv_done[q]);
-        if (j == n_kt - 1) mma_commit(&ctl.o_full[q]);
-      };
-      bool ok = mbar_wait(&ctl.q_full, 0) && mbar_wait(&ctl.k_full[0], 0);
-      if (ok) {
-        tc_fence_after();
-        for (int q = 0; q < nq; ++q) issue_s(q, 0);
-        mma_commit(&ctl.k_empty[0]);
-      }
+      const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK);
+      bool ok = mbar_wait(&ctl.q_full, 0);
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
-        const bool more = j + 1 < n_kt;
+        ok = mbar_wait(&ctl.k_full[j % kNK], (j / kNK) & 1);
+        for (int q = 0; q < nq && ok; ++q) {
+          if (j > 0) ok = mbar_wait(&ctl.pv_done[q], (j - 1) & 1);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t qaddr = aq + q * kTileBytes, kaddr = ak + (j % kNK) * kTileBytes;
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const uint32_t off = (ks >> 2) * kKSub + (ks & 3) * 32;
+            mma_ss(tS0 + q * kTN, smem_desc_sw128(qaddr + off, 16, 1024),
+                   smem_desc_sw128(kaddr + off, 16, 1024), kIdS, ks > 0);
+          }
+          mma_commit(&ctl.s_full[q]);
+        }
+        if (ok) mma_commit(&ctl.k_empty[j % kNK]);
+      }
+      if (!ok) flag_timeout(p, ctl);
+    }
+  } else if (warp == kWPv) {
+    // ------------------------------------------------------------ PV issuer
+    // O_q += P_q(j) V(j) once the softmax of tile q has stored P_q(j) and V(j) has landed.
+    if (lane == 0) {
+      constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
+      const uint32_t av = smem_u32(sV);
+      bool ok = true;
+      for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
         ok = mbar_wait(&ctl.v_full[j % kNV], (j / kNV) & 1);
-        if (ok && more) ok = mbar_wait(&ctl.k_full[(j + 1) % kNK], ((j + 1) / kNK) & 1);
         for (int q = 0; q < nq && ok; ++q) {
           ok = mbar_wait(&ctl.p_full[q], j & 1);
           if (!ok) break;
           tc_fence_after();
-          issue_pv(q, j);
-          if (q == nq - 1) mma_commit(&ctl.v_empty[j % kNV]);
-          if (more) {
-            ok = mbar_wait(&ctl.pv_done[q], j & 1);
-            if (!ok) break;
-            tc_fence_after();
-            issue_s(q, j + 1);
-            if (q == nq - 1) mma_commit(&ctl.k_empty[(j + 1) % kNK]);
-          }
+          const uint32_t vaddr = av + (j % kNV) * kTileBytes;
+#pragma unroll
+          for (int ks = 0; ks < kTN / 16; ++ks)
+            mma_ts(tO0 + q * D, tS0 + q * kTN + ks * 8,
+                   smem_desc_sw128(vaddr + ks * 2048, kKSub, 1024), kIdO,
+                   (j > 0 || ks > 0) ? 1u : 0u);
+          mma_commit(&ctl.pv_done[q]);
+          if (j == n_kt - 1) mma_commit(&ctl.o_full[q]);
         }
+        if (ok) mma_commit(&ctl.v_empty[j % kNV]);
       }
       if (!ok) flag_timeout(p, ctl);
     }

@@ -13,16 +13,17 @@
 // keys), 16 KB each, and feeds the tensor core half the operand bytes per MMA that a
 // one-CTA kernel would.
 //
-// Per CTA (352 threads, one CTA per SM, persistent over work items):
-//   warps 0-7  softmax and epilogue: warps w and w + 4 share TMEM lane quarter w (query
-//              rows 32w .. 32w + 31), each taking 64 of a tile's 128 key columns; thread 0
-//              also loads the next item's Q tile by TMA into the staging buffer;
-//   warp 8     TMA producer of this CTA's K/V halves (4 stages), L2 prefetches ahead;
-//   warp 9     TMEM allocation (both CTAs, collectively); rank 0 lane 0: S issuer;
+// Per CTA (608 threads, one CTA per SM, persistent over work items):
+//   warps 0-15 softmax and epilogue: warp w takes TMEM lane quarter w % 4 (query rows
+//              32 (w % 4) .. + 31) and key columns 32 (w / 4) .. + 31 of every tile; four
+//              warps share a row's maximum through shared memory. Thread 0 also loads the
+//              next item's Q tile by TMA into the staging buffer;
+//   warp 16    TMA producer of this CTA's K/V halves (4 stages), L2 prefetches ahead;
+//   warp 17    TMEM allocation (both CTAs, collectively); rank 0 lane 0: S issuer;
 //              rank 1 lane 0: forwards the landing of rank 1's K and V halves to rank 0's
 //              barriers (each CTA's copies complete on its own barriers, so that every
 //              CTA can wait for its own copies before it releases shared memory);
-//   warp 10    rank 0 lane 0: PV issuer.
+//   warp 18    rank 0 lane 0: PV issuer.
 //   TMEM (each CTA): S ring [0, 256) (S(t) in buffer t % 2), O [256, 384), P [384, 448)
 //   (bf16 pairs), Q [448, 512) (bf16 pairs, written by the softmax threads).
 // S = Q K^T and O += P V both take A from TMEM. Two issuer threads keep the tensor pipe
@@ -49,15 +50,19 @@
 namespace dard {
 namespace {
 
-constexpr int kPairThreads = 352;
+constexpr int kSoftmaxSlots = 4;        // softmax warps per TMEM lane quarter
+constexpr int kCols = kTN / kSoftmaxSlots;  // key columns of a tile per softmax thread
+constexpr int kSoftmaxThreads = 128 * kSoftmaxSlots;
+constexpr int kPairThreads = kSoftmaxThreads + 3 * 32;
 constexpr int kPairRows = 256;          // query rows per work item (128 per CTA)
 constexpr int kPD = 128;                // head_dim of this kernel
 constexpr int kPST = 4;                 // K/V stages (this CTA's halves)
 constexpr uint32_t kHalf = 16384;       // half of a 128-key K or V tile
 constexpr uint32_t kKBlock = 8192;      // K half: two 64-key x 64-d swizzled blocks
 constexpr uint16_t kBothCtas = 0x3;
-constexpr int kWProducer = 8, kWIssueS = 9, kWIssuePV = 10;
-constexpr int kSoftmaxArrivals = 16;    // 8 softmax warps x 2 CTAs
+constexpr int kWProducer = 4 * kSoftmaxSlots, kWIssueS = kWProducer + 1,
+              kWIssuePV = kWProducer + 2;
+constexpr int kSoftmaxArrivals = 2 * 4 * kSoftmaxSlots;  // softmax warps of both CTAs
 
 struct __align__(16) PairCtl {
   uint64_t k_land[kPST], v_land[kPST];    // this CTA's half landed (TMA bytes)
@@ -75,8 +80,8 @@ struct __align__(16) PairCtl {
   uint32_t tmem_base;
   int32_t abort;
   BlockInfo bi;
-  float red_max[2][2][128];  // per tile parity: the two column halves' row maxima
-  float red_sum[2][128];     // the two halves' row sums
+  float red_max[2][kSoftmaxSlots][128];  // per tile parity: each column slot's row maxima
+  float red_sum[kSoftmaxSlots][128];     // each column slot's row sums
   uint8_t store_row[128];    // epilogue: rows of this CTA that are written
 };
 
@@ -111,6 +116,11 @@ __device__ __forceinline__ bool bar_and(int id, int n, bool ok) {
       : "r"(static_cast<uint32_t>(ok)), "r"(id), "r"(n)
       : "memory");
   return r != 0;
+}
+
+// Named barrier 2 over every softmax thread of the CTA.
+__device__ __forceinline__ void softmax_sync() {
+  asm volatile("bar.sync 2, %0;" ::"n"(kSoftmaxThreads) : "memory");
 }
 
 __device__ __forceinline__ void pair_flag_timeout(const AttnParams& p, PairCtl& ctl) {
@@ -310,7 +320,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax + epilogue
-    const int quarter = warp & 3, half = warp >> 2;
+    // Warp w: TMEM lane quarter w % 4 (query rows 32 (w % 4) .. + 31), column slot w / 4
+    // (keys 32 slot .. + 31 of a tile, P columns 16 slot .., O and Q columns 32 slot ..).
+    const int quarter = warp & 3, slot = warp >> 2;
     const int t = quarter * 32 + lane;  // TMEM lane = this CTA's query row within the item
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const float sl = p.scale_log2;
@@ -328,24 +340,26 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         tma_load_2d(sO + kHalf, &tmq, &ctl.q_land, qi.h * D + 64, row);
       }
     };
-    // This thread's half of its query row (64 bf16: row t of block `half` of the staging
-    // buffer) into TMEM (the A-operand layout: bf16 pairs), then tell rank 0.
+    // This thread's 32 elements of its query row (d = 32 slot .., four 16-byte chunks of row
+    // t in the staging buffer's swizzled block slot / 2) into TMEM (bf16 pairs), then tell
+    // rank 0.
     auto store_q = [&]() -> bool {
       bool okq = mbar_wait(&ctl.q_land, q_loads & 1, wlim);
       okq = __all_sync(0xffffffffu, okq);
       ++q_loads;
       if (!okq) return false;
-      const uint8_t* src = sO + half * kHalf + t * 128;
-      uint32_t qw[32];
+      const uint8_t* src = sO + (slot >> 1) * kHalf + t * 128;
+      uint32_t qw[16];
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 u = *reinterpret_cast<const uint4*>(src + ((c ^ (t & 7)) << 4));
+      for (int c = 0; c < 4; ++c) {
+        const int chunk = (slot & 1) * 4 + c;
+        const uint4 u = *reinterpret_cast<const uint4*>(src + ((chunk ^ (t & 7)) << 4));
         qw[4 * c + 0] = u.x;
         qw[4 * c + 1] = u.y;
         qw[4 * c + 2] = u.z;
         qw[4 * c + 3] = u.w;
       }
-      tmem_st32(tQ + lane_off + half * 32, qw);
+      tmem_st16(tQ + lane_off + slot * 16, qw);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -361,16 +375,16 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       if (warp < 4) bf = fetch_block_info(p, p.seq[it.seq]);
       run = store_q();
     }
-    run = bar_and(2, 256, run);  // and every thread has read the staging buffer
+    run = bar_and(2, kSoftmaxThreads, run);  // and every thread has read the staging buffer
     if (run && w + ncl < p.total_pairs) load_q(pair_item(p, w + ncl));
     for (; run && w < p.total_pairs; w += ncl, ++item_it) {
-      const SeqDesc& sd = p.seq[it.seq];
+      const SeqDesc sd = p.seq[it.seq];  // a register copy: the loop reads it every tile
       const int rows_seq = sd.n_orig + sd.slen;
       const int rs = it.r0 + kBM * static_cast<int>(rank) + t;  // sequence-relative row
       // The block of this item's sequence (every softmax warp is done with the previous
       // item's copy: it passed that item's epilogue barriers).
       if (warp < 4) publish_block_info(p, sd, ctl.bi, bf, it.pr == 0 && it.h == 0 && rank == 0);
-      softmax_bar_sync();
+      softmax_sync();
       bool store_row;  // this thread's row is an output row of the call
       RowMasks rm;
       {
@@ -385,91 +399,84 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       bool ok = true;
       for (int j = 0; j < it.n_kt; ++j, ++tg) {
         const int b = tg & 1;
-        const int kt0 = j * kTN + half * 64;  // this warp's 64 keys
         const bool masked = tile_needs_mask(sd, j * kTN);
-        const uint64_t vis = masked ? vis64(sd, kt0, rm) : ~0ull;
+        const uint32_t vis =
+            masked ? static_cast<uint32_t>(vis64(sd, j * kTN + kCols * slot, rm)) : ~0u;
         bool wok = ok && !*abort_flag && mbar_wait(&ctl.s_full[b], (tg >> 1) & 1, wlim);
         wok = __all_sync(0xffffffffu, wok);
-        float s[64];
+        float s[kCols];
         float mh = -INFINITY;
         if (wok) {
           tc_fence_after();
-          uint32_t r0[32], r1[32];
-          tmem_ld32(tS + b * kTN + 64 * half + lane_off, r0);
-          tmem_ld32(tS + b * kTN + 64 * half + 32 + lane_off, r1);
+          uint32_t r[32];
+          tmem_ld32(tS + b * kTN + kCols * slot + lane_off, r);
           tmem_wait_ld();
           // S(t) is in registers: rank 0 may reuse its buffer for S(t + 2)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive_remote(lead(&ctl.s_free[b]));
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            s[e] = __uint_as_float(r0[e]);
-            s[32 + e] = __uint_as_float(r1[e]);
-          }
+          for (int e = 0; e < 32; ++e) s[e] = __uint_as_float(r[e]);
           if (masked) {
 #pragma unroll
-            for (int k = 0; k < 64; ++k) s[k] = ((vis >> k) & 1ull) ? s[k] : -INFINITY;
+            for (int k = 0; k < 32; ++k) s[k] = ((vis >> k) & 1u) ? s[k] : -INFINITY;
           }
           float mx[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) mx[e] = fmax3(s[e], s[8 + e], s[16 + e]);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) mx[e] = fmax3(mx[e], s[24 + e], s[32 + e]);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) mx[e] = fmax3(mx[e], s[40 + e], s[48 + e]);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[56 + e]);
+          for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[24 + e]);
           mh = fmaxf(fmax3(mx[0], mx[1], mx[2]), fmax3(fmax3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
-          ctl.red_max[tg & 1][half][t] = mh;
+          ctl.red_max[tg & 1][slot][t] = mh;
         }
-        // both warps of the row leave together, or both go on with both maxima
-        if (!bar_and(3 + quarter, 64, wok)) {
+        // the four warps of the rows leave together, or all go on with all four maxima
+        if (!bar_and(3 + quarter, 32 * kSoftmaxSlots, wok)) {
           ok = false;
           break;
         }
-        const float mt = fmaxf(mh, ctl.red_max[tg & 1][half ^ 1][t]);
+        const float mt = fmaxf(fmaxf(ctl.red_max[tg & 1][0][t], ctl.red_max[tg & 1][1][t]),
+                               fmaxf(ctl.red_max[tg & 1][2][t], ctl.red_max[tg & 1][3][t]));
         // Raise the reference maximum on the first finite value, or when the tile maximum
         // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
-        // Both warps of a row take the same decision from the same values.
+        // The four warps of a row take the same decision from the same values.
         float m_new = m_run;
         if (m_run == -INFINITY) m_new = mt;
         else if ((mt - m_run) * sl > kRescaleLog2) m_new = mt;
         const bool rescale = (m_new != m_run) && (m_run != -INFINITY);
         const float alpha = rescale ? ex2_approx((m_run - m_new) * sl) : 1.f;
         const float mL = (m_new == -INFINITY) ? 0.f : m_new * sl;
-        uint32_t pk[32];
+        uint32_t pk[16];
         const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
-        uint64_t acc[4] = {0, 0, 0, 0};  // four packed partial sums (bit pattern 0 = +0.0f)
+        uint64_t acc[2] = {0, 0};  // two packed partial sums (bit pattern 0 = +0.0f)
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
+        for (int e = 0; e < 16; ++e) {
           float x0, x1;
           f2_unpack(f2_fma(f2_pack(s[2 * e], s[2 * e + 1]), sl2, nmL2), x0, x1);
           pk[e] = pack_bf16x2(ex2_approx(x0), ex2_approx(x1));
           // the row sum adds the rounded weights the PV product multiplies with
-          acc[e & 3] = f2_add(acc[e & 3], f2_pack(__uint_as_float(pk[e] << 16),
+          acc[e & 1] = f2_add(acc[e & 1], f2_pack(__uint_as_float(pk[e] << 16),
                                                   __uint_as_float(pk[e] & 0xffff0000u)));
         }
-        float a0, a1, c0, c1;
+        float a0, a1;
         f2_unpack(f2_add(acc[0], acc[1]), a0, a1);
-        f2_unpack(f2_add(acc[2], acc[3]), c0, c1);
         // P(t) replaces P(t - 1), and O may be rescaled, once PV(t - 1) has completed
         wok = tg == 0 || mbar_wait(&ctl.pv_done, (tg - 1) & 1, wlim);
         wok = __all_sync(0xffffffffu, wok);
         if (!wok) {
-          // leave with the partner at the next tile's barrier (or the epilogue's)
+          // leave with the other warps of the rows at the next tile's barrier (or the
+          // epilogue's)
           ok = false;
           continue;
         }
         tc_fence_after();
-        tmem_st32(tP + lane_off + 32 * half, pk);
+        tmem_st16(tP + lane_off + 16 * slot, pk);
         // O (stable: PV(t - 1) completed, PV(t) waits for the arrival below) is rescaled
         // only when the reference maximum moved
         if (__any_sync(0xffffffffu, rescale)) {
 #pragma unroll 1
-          for (int c = 0; c < 4; ++c) {  // this warp's half of the O columns
+          for (int c = 0; c < 2; ++c) {  // this warp's 32 O columns
             uint32_t r[16];
-            const uint32_t col = tO + lane_off + half * 64 + 16 * c;
+            const uint32_t col = tO + lane_off + kCols * slot + 16 * c;
             tmem_ld16(col, r);
             tmem_wait_ld();
 #pragma unroll
@@ -477,7 +484,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
             tmem_st16(col, r);
           }
         }
-        l_run = l_run * alpha + ((a0 + a1) + (c0 + c1));
+        l_run = l_run * alpha + (a0 + a1);
         m_run = m_new;
         tmem_wait_st();
         tc_fence_before();
@@ -491,42 +498,40 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       // ---------------------------------------------------------- epilogue
       bool wok = ok && mbar_wait(&ctl.o_full, item_it & 1, wlim);
       wok = __all_sync(0xffffffffu, wok);
-      ctl.red_sum[half][t] = l_run;
-      const bool all_ok = bar_and(2, 256, wok);  // every softmax warp's verdict, and sync
+      ctl.red_sum[slot][t] = l_run;
+      const bool all_ok = bar_and(2, kSoftmaxThreads, wok);  // every warp's verdict, and sync
       if (!all_ok && lane == 0 && !wok) pair_flag_timeout(p, ctl);
       constexpr int kChunks = D / 8;  // 16-byte chunks per output row
       uint4* stage = reinterpret_cast<uint4*>(sO);
       if (all_ok) {
         tc_fence_after();
-        const float inv_l = 1.0f / (ctl.red_sum[0][t] + ctl.red_sum[1][t]);
+        const float inv_l =
+            1.0f / ((ctl.red_sum[0][t] + ctl.red_sum[1][t]) + (ctl.red_sum[2][t] + ctl.red_sum[3][t]));
+        uint32_t rr[32];
+        tmem_ld32(tO + lane_off + kCols * slot, rr);
+        tmem_wait_ld();
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          uint32_t rr[32];
-          tmem_ld32(tO + lane_off + half * 64 + 32 * c, rr);
-          tmem_wait_ld();
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            uint4 u;
-            u.x = pack_bf16x2(__uint_as_float(rr[8 * v + 0]) * inv_l, __uint_as_float(rr[8 * v + 1]) * inv_l);
-            u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
-            u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
-            u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
-            const int chunk = half * (kChunks / 2) + c * 4 + v;
-            stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
-          }
+        for (int v = 0; v < 4; ++v) {
+          uint4 u;
+          u.x = pack_bf16x2(__uint_as_float(rr[8 * v + 0]) * inv_l, __uint_as_float(rr[8 * v + 1]) * inv_l);
+          u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
+          u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
+          u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
+          const int chunk = slot * 4 + v;
+          stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
         }
         // O has been read out: rank 0 may start the next item's first PV
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_remote(lead(&ctl.o_free));
       }
-      if (half == 0) ctl.store_row[t] = (all_ok && store_row) ? 1 : 0;
-      softmax_bar_sync();
+      if (slot == 0) ctl.store_row[t] = (all_ok && store_row) ? 1 : 0;
+      softmax_sync();
       if (all_ok) {
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.o);
         const size_t rbase = static_cast<size_t>(sd.row_base) + it.r0 + kBM * rank;
 #pragma unroll 4
-        for (int idx = threadIdx.x; idx < kBM * kChunks; idx += 256) {
+        for (int idx = threadIdx.x; idx < kBM * kChunks; idx += kSoftmaxThreads) {
           const int row = idx / kChunks, chunk = idx % kChunks;
           if (ctl.store_row[row]) {
             const uint4 u = stage[row * kChunks + (chunk ^ (row & (kChunks - 1)))];
@@ -536,7 +541,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         }
       }
       // the staging buffer takes the next Q tile only after every thread has stored from it
-      const bool cont = bar_and(2, 256, all_ok && go_on);
+      const bool cont = bar_and(2, kSoftmaxThreads, all_ok && go_on);
       if (!cont) break;
       if (w + 2 * ncl < p.total_pairs) load_q(pair_item(p, w + 2 * ncl));
       it = pair_item(p, w + ncl);
