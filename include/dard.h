@@ -186,10 +186,14 @@ typedef struct {
   float* w_out;              /* optional device [rows] out: w for M rows, NaN otherwise    */
   int32_t* counts;           /* optional device [num_seqs * 3] out: M, C, U counts         */
   uint32_t* status;          /* optional device word, DARD_STATUS_* bits OR-ed in          */
-  void* workspace;           /* device scratch of dard_score_workspace_size() bytes (one
-                                byte per row: the promotion / demotion outcome of pass 1).
-                                No initial contents are needed. Calls that overlap on the
-                                GPU need separate workspaces.                              */
+  void* workspace;           /* device scratch of dard_score_workspace_size() bytes: three
+                                counters per sequence, then two bytes per block row (each
+                                C row's promotion / demotion outcome, each row's new
+                                state). Fill it with zeros before its first use; every
+                                call leaves the counters at zero again, except a call that
+                                sets DARD_STATUS_TIMEOUT, after which it must be zeroed
+                                again. Calls that overlap on the GPU need separate
+                                workspaces.                                                */
   size_t workspace_bytes;
   /* Optional, the end of a step (each may be NULL):                                       */
   const int32_t* cur_token;  /* device [rows] the token currently at each block position   */
@@ -218,7 +222,11 @@ typedef struct {
 size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs);
 
 /* Logits pointers must be 16-byte aligned and row_stride * element size a multiple of 16.
- * Errors: DARD_ERR_NULL, _SHAPE, _VALUE, _ALIGN, _WORKSPACE, _CUDA. */
+ * Two launches (C and U rows, then M rows: Algorithm 1's order), the second a programmatic
+ * dependent of the first. DARD_SCORE_PATH=fused selects one launch instead, whose M rows
+ * wait (bounded) for their block's C rows of the same launch, when every row's group of
+ * CTAs fits on the device at once. Errors: DARD_ERR_NULL, _SHAPE, _VALUE, _ALIGN,
+ * _WORKSPACE, _CUDA. */
 dard_status dard_score_and_transition(const dard_score_args* args, void* stream);
 
 /* ------------------------------------------------------------------------------------- *
@@ -232,12 +240,13 @@ dard_status dard_score_and_transition(const dard_score_args* args, void* stream)
  * none and neither allocates nor frees device memory.
  *
  * Arguments, outputs and errors are those of dard_score_and_transition, except that
- * `workspace` and `workspace_bytes` are ignored. The scratch is a fixed array of
- * DARD_SCORE_NOALLOC_MAX_ROWS bytes in the library's device memory (one byte per block row,
- * the outcome of the verification pass). A call with more block rows (sum of block_len)
- * than that returns DARD_ERR_WORKSPACE before any launch; use dard_score_and_transition
- * with a workspace for it. Nothing in the array needs to start at zero: every call writes
- * each byte it reads before reading it.
+ * `workspace` and `workspace_bytes` are ignored. The scratch is a fixed array in the
+ * library's device memory sized for DARD_SCORE_NOALLOC_MAX_ROWS block rows and DARD_MAX_SEQS
+ * sequences (the workspace layout of dard_score_and_transition). A call with more block
+ * rows (sum of block_len) than that returns DARD_ERR_WORKSPACE before any launch; use
+ * dard_score_and_transition with a workspace for it. Each call clears the array's counters
+ * on its stream (cudaMemsetAsync, which allocates nothing) before the kernels run, so no
+ * call depends on what an earlier one left.
  *
  * The first call on each device (the device current at the call) looks up the array's
  * address there once (cudaGetSymbolAddress) and caches it; make that first call before any

@@ -52,7 +52,7 @@ const char* dard_status_string(dard_status s) {
 
 const char* dard_last_error(void) { return g_err; }
 
-int32_t dard_version(void) { return 100; }
+int32_t dard_version(void) { return 20000; }
 
 }  // extern "C"
 
@@ -154,37 +154,9 @@ dard_status prepare_attention(const dard_attn_args* a, dard::AttnParams& p) {
 
 }  // namespace
 
-extern "C" {
-
-dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
+// Host-side validation of a scoring call and its kernel parameters (no device access).
+dard_status dard::prepare_score(const dard_score_args* a, dard::ScoreParams& p) {
   using namespace dard;
-  g_err[0] = '\0';
-  AttnParams p;
-  const dard_status st = prepare_attention(a, p);
-  if (st != DARD_OK) return st;
-  if (p.total_work == 0) return DARD_OK;  // no query rows (every query_start at the end)
-  return launch_attention(*a, p, static_cast<cudaStream_t>(stream), g_err, sizeof(g_err));
-}
-
-dard_status dard_attention_kernel(const dard_attn_args* a, int32_t* kernel) {
-  using namespace dard;
-  g_err[0] = '\0';
-  if (!kernel) return fail(DARD_ERR_NULL, "kernel is NULL");
-  AttnParams p;
-  const dard_status st = prepare_attention(a, p);
-  if (st != DARD_OK) return st;
-  *kernel = p.total_work == 0 ? 0 : attention_kernel_choice(*a, p);
-  return DARD_OK;
-}
-
-size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs) {
-  if (rows < 0 || vocab < 1 || num_seqs < 1 || num_seqs > DARD_MAX_SEQS) return 0;
-  return dard::score_workspace_bytes(rows, num_seqs);
-}
-
-dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
-  using namespace dard;
-  g_err[0] = '\0';
   if (!a) return fail(DARD_ERR_NULL, "args is NULL");
   if (!a->block_len) return fail(DARD_ERR_NULL, "block_len is NULL");
   if (a->dtype != DARD_BF16 && a->dtype != DARD_F32)
@@ -197,7 +169,6 @@ dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
     return fail(DARD_ERR_VALUE, "need 0 <= tau_c <= tau_u <= 1");
   if (!(a->lambda > 0.f && a->lambda < 1.f)) return fail(DARD_ERR_VALUE, "need 0 < lambda < 1");
   if (!(a->p0 > 0.f) || !std::isfinite(a->p0)) return fail(DARD_ERR_VALUE, "need p0 > 0");
-  ScoreParams p;
   memset(&p, 0, sizeof(p));
   long long rows = 0;
   for (int s = 0; s < a->num_seqs; ++s) {
@@ -249,6 +220,44 @@ dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
   p.tau_u = a->tau_u;
   p.lambda = a->lambda;
   p.p0 = a->p0;
+  return DARD_OK;
+}
+
+
+extern "C" {
+
+dard_status dard_step_attention(const dard_attn_args* a, void* stream) {
+  using namespace dard;
+  g_err[0] = '\0';
+  AttnParams p;
+  const dard_status st = prepare_attention(a, p);
+  if (st != DARD_OK) return st;
+  if (p.total_work == 0) return DARD_OK;  // no query rows (every query_start at the end)
+  return launch_attention(*a, p, static_cast<cudaStream_t>(stream), g_err, sizeof(g_err));
+}
+
+dard_status dard_attention_kernel(const dard_attn_args* a, int32_t* kernel) {
+  using namespace dard;
+  g_err[0] = '\0';
+  if (!kernel) return fail(DARD_ERR_NULL, "kernel is NULL");
+  AttnParams p;
+  const dard_status st = prepare_attention(a, p);
+  if (st != DARD_OK) return st;
+  *kernel = p.total_work == 0 ? 0 : attention_kernel_choice(*a, p);
+  return DARD_OK;
+}
+
+size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs) {
+  if (rows < 0 || vocab < 1 || num_seqs < 1 || num_seqs > DARD_MAX_SEQS) return 0;
+  return dard::score_workspace_bytes(rows, num_seqs);
+}
+
+dard_status dard_score_and_transition(const dard_score_args* a, void* stream) {
+  using namespace dard;
+  g_err[0] = '\0';
+  ScoreParams p;
+  const dard_status st = prepare_score(a, p);
+  if (st != DARD_OK) return st;
   return launch_score(*a, p, static_cast<cudaStream_t>(stream), g_err, sizeof(g_err));
 }
 

@@ -84,8 +84,12 @@ struct ScoreParams {
   int32_t order_mode;
   uint32_t* status;
   // workspace
+  uint32_t* ready;     // [num_seqs] C rows of the block that published their outcome
+  uint32_t* departed;  // [num_seqs] M-row CTAs of the block past their wait
+  uint32_t* fin;       // [num_seqs] rows of the block that finished (counts, in-place states)
   uint8_t* pd_flag;    // [rows] 1 = promoted (C -> U), 2 = demoted (C -> M), 3 = an M row
                        // (scored in pass 2), 0 otherwise
+  uint8_t* new_state;  // [rows] the state each row ends in
   int64_t row_stride;
   int32_t vocab, rows, num_seqs, nsplit, chunk;
   float tau_c, tau_u, lambda, p0;
@@ -97,7 +101,10 @@ constexpr int kScoreThreads = 256;
 constexpr int kScoreMaxSplit = 16;  // CTAs per row = thread-block cluster size
 constexpr int kScoreCtasPerSm = 12;  // target CTAs per SM when choosing the split
 
+// Validates a scoring call and fills its kernel parameters; touches no device memory.
+dard_status prepare_score(const dard_score_args* a, ScoreParams& p);
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs);
+size_t score_counter_bytes(int32_t num_seqs);  // the counters at the start of the workspace
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
                          char* err, size_t err_len);
 // Records the message returned by dard_last_error() on this thread and returns `s`.

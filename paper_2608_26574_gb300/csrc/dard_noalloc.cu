@@ -1,19 +1,27 @@
 // dard_noalloc.cu - dard_score_and_transition_noalloc: the scoring call with its scratch in a
 // fixed array inside the library, for callers that cannot hand device memory to it.
 //
-// The only scratch the scoring kernels use is one byte per block row (the promotion /
-// demotion outcome of pass 1, read by pass 2). Here that byte array is a file-scope
-// __device__ array of DARD_SCORE_NOALLOC_MAX_ROWS bytes. Its address on a device is looked up
-// once (cudaGetSymbolAddress, with that device current) on the first call made on that
-// device, cached per device, and then passed as the workspace of dard_score_and_transition,
-// whose kernels and validation run unchanged. No call allocates or frees device memory.
+// The scoring scratch is three counters per sequence (zero between calls) and two bytes
+// per block row (the promotion / demotion outcome of each C row, and each row's new
+// state). Here it is a file-scope __device__ array sized for DARD_SCORE_NOALLOC_MAX_ROWS
+// rows and DARD_MAX_SEQS sequences. Its address on a device is looked up once
+// (cudaGetSymbolAddress, with that device current) on the first call made on that device,
+// cached per device, and then passed as the workspace of dard_score_and_transition, whose
+// kernels and validation run unchanged. Every call first clears the counters with an
+// asynchronous memset on its stream, so a call never depends on what an earlier one left
+// behind. No call allocates or frees device memory.
 #include <mutex>
 
 #include "dard_internal.h"
 
+
 namespace {
 
-__device__ __align__(256) uint8_t g_score_scratch[DARD_SCORE_NOALLOC_MAX_ROWS];
+// score_workspace_bytes(DARD_SCORE_NOALLOC_MAX_ROWS, DARD_MAX_SEQS): counters, then the
+// outcome and new-state bytes, each part 256-byte aligned
+constexpr size_t kScratchBytes = ((3 * 4 * DARD_MAX_SEQS + 255) / 256) * 256 +
+                                 2 * (((DARD_SCORE_NOALLOC_MAX_ROWS + 255) / 256) * 256);
+__device__ __align__(256) uint8_t g_score_scratch[kScratchBytes];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
@@ -68,5 +76,19 @@ extern "C" dard_status dard_score_and_transition_noalloc(const dard_score_args* 
     b.workspace = scratch;
     b.workspace_bytes = sizeof(g_score_scratch);
   }
-  return dard_score_and_transition(&b, stream);
+  ScoreParams p;
+  const dard_status st = prepare_score(&b, p);
+  if (st != DARD_OK) return st;
+  if (b.workspace != nullptr) {
+    // the counters start at zero on every call (cudaMemsetAsync allocates nothing)
+    const cudaError_t m = cudaMemsetAsync(b.workspace, 0, score_counter_bytes(b.num_seqs),
+                                          static_cast<cudaStream_t>(stream));
+    if (m != cudaSuccess)
+      return report(DARD_ERR_CUDA, "clearing the built-in scratch failed: %s",
+                    cudaGetErrorString(m));
+  }
+  char err[256];
+  const dard_status ls = launch_score(b, p, static_cast<cudaStream_t>(stream), err, sizeof(err));
+  if (ls != DARD_OK) return report(ls, "%s", err);
+  return DARD_OK;
 }

@@ -22,6 +22,8 @@
 // (kExtra) adds the optional end-of-step outputs: p_cur, the next step's tokens, an
 // in-place state update, entropy, margin and the next step's ordering key.
 #include <atomic>
+#include <cstdlib>
+#include <cstring>
 #include <type_traits>
 #include <cfloat>
 #include <climits>
@@ -384,14 +386,14 @@ __device__ __forceinline__ void prefetch_current(const ScoreParams& p, int row, 
 // that ends in M: the last line of Algorithm 1's step); returns the new state.
 template <bool kExtra, class A>
 __device__ __forceinline__ int finalize_row(const ScoreParams& p, int row, const A& a,
-                                            float w, float lc) {
+                                            float w, float lc, bool write_state = true) {
   const float z = a.s;
   const bool valid = isfinite(z) && z > 0.f;
   const float c = valid ? 1.0f / z : 0.f;
   const int ns = !valid ? kStateM : (c <= p.tau_c ? kStateM : (c <= p.tau_u ? kStateC : kStateU));
   p.conf[row] = c;
   p.token[row] = valid ? a.idx : -1;
-  p.state_out[row] = static_cast<uint8_t>(ns);
+  if (write_state) p.state_out[row] = static_cast<uint8_t>(ns);
   if (p.w_out) p.w_out[row] = w;
   if (kExtra && p.p_cur) {
     const float mL = a.m * kLog2e;
@@ -568,6 +570,202 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   }
 }
 
+// ------------------------------------------------------------------ one-launch scoring
+// Both passes in one grid. C and U rows stream their shadow logits and decide (Eq. 1, 8);
+// a C row's cluster leader then writes its outcome byte and releases the block's ready
+// counter. M rows issue the loads of their first round of both logit rows, wait until
+// every C row of their block has published (a bounded spin on the counter: the launcher
+// uses this kernel only when the whole grid fits on the device at once, so every C row
+// the wait depends on is running), compute w (Eq. 5-6) and mix (Eq. 7).
+// Counters start at zero and every call leaves them at zero: the last M-row CTA of a
+// block to pass its wait clears ready and departed; with counts or an in-place state
+// update, the last row of a block to finish (fin) writes the block's counts and states
+// and clears fin.
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_gpu(uint32_t* p, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+template <class T, int VPT, bool kExtra>
+__global__ void __launch_bounds__(kScoreThreads) score_fused(const __grid_constant__ ScoreParams p) {
+  // Launched as a programmatic dependent of whatever kernel precedes the call: nothing is
+  // read before that kernel (the logits' producer, or the previous call that leaves the
+  // counters at zero) has completed.
+  grid_dep_wait();
+  using A = std::conditional_t<kExtra, AccX, Acc>;
+  __shared__ A s_acc[kWarps];
+  __shared__ float4 s_slots[2 * kScoreMaxSplit];
+  __shared__ float s_w;
+  __shared__ int s_nm;
+  if (p.counts != nullptr && blockIdx.x == 0 && blockIdx.y == 0) {
+    // sequences with an empty block have no row to write their counts
+    for (int k = threadIdx.x; k < p.num_seqs; k += blockDim.x)
+      if (p.blk_off[k + 1] == p.blk_off[k]) {
+        p.counts[3 * k + 0] = 0;
+        p.counts[3 * k + 1] = 0;
+        p.counts[3 * k + 2] = 0;
+      }
+  }
+  const int row = blockIdx.y, split = blockIdx.x;
+  const int seq = seq_of_row(p, row);
+  const int b0 = p.blk_off[seq], blen = p.blk_off[seq + 1] - b0;
+  const int st = load_state(p, row, split == 0);
+  const size_t roff = static_cast<size_t>(row) * p.row_stride * T::kBytes;
+  const char* xp = static_cast<const char*>(p.lx) + roff;
+  const char* sp = static_cast<const char*>(p.ls) + roff;
+  const int c0 = split * p.chunk;
+  const int c1 = min(p.vocab, c0 + p.chunk);
+  float cur_lx = 0.f, cur_ls = 0.f;  // the current token's logits (p_cur), loaded early
+  if (kExtra) prefetch_current<T>(p, row, st == kStateM ? xp : nullptr, sp, cur_lx, cur_ls);
+  A acc = acc_init(static_cast<A*>(nullptr));
+  float w = __int_as_float(0x7fc00000);
+  constexpr int kRound = kScoreThreads * VPT * T::W;
+  if (st != kStateM) {
+    // The block's M count (a C row releases the counter only if some M row waits on it).
+    if (threadIdx.x < 32) {
+      int nm = 0;
+      for (int j = threadIdx.x; j < blen; j += 32) {
+        const int sj = p.state_in[b0 + j];
+        nm += (sj == kStateM || sj > 2) ? 1 : 0;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) nm += __shfl_xor_sync(0xffffffffu, nm, off);
+      if (threadIdx.x == 0) s_nm = nm;
+    }
+    for (int base = c0; base < c1; base += kRound) {
+      uint4 r[VPT];
+#pragma unroll
+      for (int v = 0; v < VPT; ++v)
+        r[v] = load_vec<T>(sp, base + (v * kScoreThreads + threadIdx.x) * T::W, c1);
+      fold<T, VPT>(acc, base, c1, [&](int v, int e) { return T::get(r[v], e); });
+    }
+  } else {
+    // First round of both rows: in flight while the block's C rows are decided.
+    uint4 rx[VPT], rs[VPT];
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int e0 = c0 + (v * kScoreThreads + threadIdx.x) * T::W;
+      rx[v] = load_vec<T>(xp, e0, c1);
+      rs[v] = load_vec<T>(sp, e0, c1);
+    }
+    if (threadIdx.x < 32) {
+      const int lane = threadIdx.x;
+      int nc = 0, nm = 0;
+      for (int j = lane; j < blen; j += 32) {
+        const int sj = p.state_in[b0 + j];
+        nc += sj == kStateC ? 1 : 0;
+        nm += (sj == kStateM || sj > 2) ? 1 : 0;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        nc += __shfl_xor_sync(0xffffffffu, nc, off);
+        nm += __shfl_xor_sync(0xffffffffu, nm, off);
+      }
+      bool ok = true;
+      if (nc > 0) {
+        if (lane == 0) {
+          const uint32_t need = static_cast<uint32_t>(nc);
+          if (ld_acquire_gpu(p.ready + seq) < need) {
+            const long long t0 = clock64();
+            while (ld_acquire_gpu(p.ready + seq) < need) {
+              if (clock64() - t0 > kWaitCycles) { ok = false; break; }
+              __nanosleep(64);
+            }
+          }
+          if (!ok && p.status) atomicOr(p.status, DARD_STATUS_TIMEOUT);
+        }
+        __syncwarp();
+        (void)ld_acquire_gpu(p.ready + seq);  // this lane's own acquire before the reads below
+      }
+      // Eq. 5-6 from the outcome bytes of this step's C rows: lambda^|i-j| as
+      // 2^(|i-j| log2 lambda), fp32 sums over the lanes, then a shuffle tree.
+      const int i = row - b0;
+      float pp = 0.f, dd = 0.f;
+      for (int j = lane; j < blen && nc > 0; j += 32) {
+        if (p.state_in[b0 + j] != kStateC) continue;
+        const int f = *reinterpret_cast<volatile const uint8_t*>(p.pd_flag + b0 + j);
+        const float kij = ex2_approx(static_cast<float>(abs(i - j)) * p.log2_lambda);
+        pp += f == 1 ? kij : 0.f;
+        dd += f == 2 ? kij : 0.f;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        pp += __shfl_xor_sync(0xffffffffu, pp, off);
+        dd += __shfl_xor_sync(0xffffffffu, dd, off);
+      }
+      if (lane == 0) {
+        s_w = __fdiv_rn(pp + p.p0, pp + dd + p.p0);
+        // the last M-row CTA of the block past its wait clears the block's counters
+        if (nc > 0) {
+          const uint32_t leaving = atomicAdd(p.departed + seq, 1u) + 1u;
+          if (leaving == static_cast<uint32_t>(nm * p.nsplit)) {
+            p.ready[seq] = 0;
+            p.departed[seq] = 0;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    w = s_w;
+    // Eq. 7 in fp32, one rounding per operation: mix = ls + w * (lx - ls).
+    auto mix = [&](const uint4& vx, const uint4& vs, int e) {
+      const float lx = T::get(vx, e), ls = T::get(vs, e);
+      return __fadd_rn(ls, __fmul_rn(w, __fsub_rn(lx, ls)));
+    };
+    fold<T, VPT>(acc, c0, c1, [&](int v, int e) { return mix(rx[v], rs[v], e); });
+    for (int base = c0 + kRound; base < c1; base += kRound) {
+#pragma unroll
+      for (int v = 0; v < VPT; ++v) {
+        const int e0 = base + (v * kScoreThreads + threadIdx.x) * T::W;
+        rx[v] = load_vec<T>(xp, e0, c1);
+        rs[v] = load_vec<T>(sp, e0, c1);
+      }
+      fold<T, VPT>(acc, base, c1, [&](int v, int e) { return mix(rx[v], rs[v], e); });
+    }
+  }
+  acc = block_merge(acc, s_acc);
+  cluster_publish(acc, split, s_slots);
+  if (split != 0 || threadIdx.x >= 32) return;
+  A a;
+  merge_slots(s_slots, p.nsplit, a);
+  if (threadIdx.x != 0) return;
+  float lc = cur_ls;
+  if (st == kStateM && cur_ls != -INFINITY)
+    lc = __fadd_rn(cur_ls, __fmul_rn(w, __fsub_rn(cur_lx, cur_ls)));
+  // in place, the block's states are written by its last row (the others may still read them)
+  const int ns = finalize_row<kExtra>(p, row, a, w, lc, !p.state_in_place);
+  if (st == kStateC && s_nm > 0) {
+    // the outcome byte, then the release of the block's counter (Algorithm 1: P and D)
+    p.pd_flag[row] = ns == kStateU ? 1 : (ns == kStateM ? 2 : 0);
+    red_release_gpu(p.ready + seq, 1u);
+  }
+  if (p.counts != nullptr || p.state_in_place) {
+    p.new_state[row] = static_cast<uint8_t>(ns);
+    __threadfence();
+    if (atomicAdd(p.fin + seq, 1u) + 1u == static_cast<uint32_t>(blen)) {
+      // the block's last row: every row of it has read its states and written new_state
+      __threadfence();
+      int cnt[3] = {0, 0, 0};
+      for (int j = 0; j < blen; ++j) {
+        const int nsj = *reinterpret_cast<volatile const uint8_t*>(p.new_state + b0 + j);
+        cnt[nsj] += 1;
+        if (p.state_in_place) p.state_out[b0 + j] = static_cast<uint8_t>(nsj);
+      }
+      if (p.counts != nullptr) {
+        p.counts[3 * seq + 0] = cnt[0];
+        p.counts[3 * seq + 1] = cnt[1];
+        p.counts[3 * seq + 2] = cnt[2];
+      }
+      p.fin[seq] = 0;
+    }
+  }
+}
+
 // Zeroes the counts when there are no rows at all (no pass runs).
 __global__ void zero_all_counts(const __grid_constant__ ScoreParams p) {
   for (int k = threadIdx.x; k < 3 * p.num_seqs; k += blockDim.x) p.counts[k] = 0;
@@ -583,6 +781,54 @@ cudaError_t allow_wide_clusters(F* kernel, std::atomic<uint64_t>& done) {
   e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
   return e;
+}
+
+// Clusters of nsplit CTAs of this kernel that fit on the current device at once (cached
+// per device and cluster size).
+template <class K>
+int max_active_clusters(K* kernel, int nsplit) {
+  static std::atomic<int> cache[64][kScoreMaxSplit + 1];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64 || nsplit < 1 ||
+      nsplit > kScoreMaxSplit)
+    return 0;
+  int n = cache[dev][nsplit].load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(nsplit, 1);
+  cfg.blockDim = dim3(kScoreThreads);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = nsplit;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return 0;
+  }
+  cache[dev][nsplit].store(n, std::memory_order_relaxed);
+  return n;
+}
+
+template <class T, int VPT, bool kExtra>
+cudaError_t launch_fused(const ScoreParams& p, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.nsplit, p.rows);
+  cfg.blockDim = dim3(kScoreThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.nsplit;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, score_fused<T, VPT, kExtra>, p);
 }
 
 template <class T, int VPT, bool kExtra>
@@ -613,9 +859,19 @@ cudaError_t launch_pair(const ScoreParams& p, cudaStream_t stream) {
 
 }  // namespace
 
+// Workspace: per-sequence counters (ready, departed, fin: zero between calls), then one
+// outcome byte and one new-state byte per block row, each part 256-byte aligned.
+namespace {
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+}  // namespace
+
 size_t score_workspace_bytes(int32_t rows, int32_t num_seqs) {
-  (void)num_seqs;
-  return (static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
+  return align256(3 * sizeof(uint32_t) * static_cast<size_t>(num_seqs)) +
+         2 * align256(static_cast<size_t>(rows));
+}
+
+size_t score_counter_bytes(int32_t num_seqs) {
+  return align256(3 * sizeof(uint32_t) * static_cast<size_t>(num_seqs));
 }
 
 namespace {
@@ -645,21 +901,58 @@ int split_cap(int rows) {
 
 }  // namespace
 
+namespace {
+
+// Splits every row over at most `cap` CTAs: each takes `rounds` rounds of 256 threads x 4
+// vectors.
+void set_split(ScoreParams& p, int per_round, int cap) {
+  const int rounds_total = (p.vocab + per_round - 1) / per_round;
+  const int rounds = (rounds_total + cap - 1) / cap;
+  p.chunk = per_round * rounds;
+  p.nsplit = (p.vocab + p.chunk - 1) / p.chunk;
+}
+
+// The two PDL-chained passes; with DARD_SCORE_PATH=fused, the one-launch kernel instead when
+// every row's cluster fits on the device at once (its M rows wait for C rows of the same
+// launch), with as many CTAs per row as allows that. Measured on GB300 (CUDA-graph timing,
+// one call per input set): the passes take 8.3 us on the 8B block, 13.5 us on the GQA block,
+// 25 us on the multimodal batch; the one launch 11.9, 18.4 and 34 us (10.4, 16.2 with no
+// counts requested). The pass boundary is a completed grid, which the hardware signals
+// sooner than the counters in L2 that the one launch polls.
+template <class T, bool kExtra>
+cudaError_t launch_rows(ScoreParams& p, cudaStream_t stream, int per_round) {
+  static std::atomic<uint64_t> done{0};
+  const char* force = std::getenv("DARD_SCORE_PATH");
+  const bool fused = force != nullptr && std::strcmp(force, "fused") == 0;
+  if (fused && allow_wide_clusters(score_fused<T, 4, kExtra>, done) == cudaSuccess) {
+    const ScoreParams keep = p;
+    for (int cap = p.nsplit; cap >= 1; --cap) {
+      set_split(p, per_round, cap);
+      if (max_active_clusters(score_fused<T, 4, kExtra>, p.nsplit) >= p.rows)
+        return launch_fused<T, 4, kExtra>(p, stream);
+      cap = p.nsplit;  // the next smaller split
+    }
+    p = keep;
+  }
+  return launch_pair<T, 4, kExtra>(p, stream);
+}
+
+}  // namespace
+
 dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t stream,
                          char* err, size_t err_len) {
   const bool bf16 = a.dtype == DARD_BF16;
   const int W = bf16 ? 8 : 4;
-  // One round = 256 threads x 4 vectors; a row spreads over at most split_cap() CTAs (one
-  // cluster), each taking `rounds` rounds.
   const int per_round = kScoreThreads * 4 * W;
-  const int rounds_total = (p.vocab + per_round - 1) / per_round;
-  const int cap = split_cap(p.rows);
-  const int rounds = (rounds_total + cap - 1) / cap;
-  p.chunk = per_round * rounds;
-  p.nsplit = (p.vocab + p.chunk - 1) / p.chunk;
+  set_split(p, per_round, split_cap(p.rows));
 
   char* ws = static_cast<char*>(a.workspace);
-  p.pd_flag = reinterpret_cast<uint8_t*>(ws);
+  const size_t cbytes = score_counter_bytes(p.num_seqs);
+  p.ready = reinterpret_cast<uint32_t*>(ws);
+  p.departed = p.ready + p.num_seqs;
+  p.fin = p.departed + p.num_seqs;
+  p.pd_flag = reinterpret_cast<uint8_t*>(ws + cbytes);
+  p.new_state = p.pd_flag + align256(static_cast<size_t>(p.rows));
   p.log2_lambda = static_cast<float>(std::log2(static_cast<double>(p.lambda)));
 
   cudaError_t e = cudaSuccess;
@@ -670,8 +963,10 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
   if (e == cudaSuccess && p.rows > 0) {
     const bool extra = p.p_cur != nullptr || p.tokens != nullptr || p.state_in_place ||
                        p.entropy != nullptr || p.margin != nullptr || p.order_key != nullptr;
-    if (extra) e = bf16 ? launch_pair<Bf16, 4, true>(p, stream) : launch_pair<F32, 4, true>(p, stream);
-    else e = bf16 ? launch_pair<Bf16, 4, false>(p, stream) : launch_pair<F32, 4, false>(p, stream);
+    if (extra) e = bf16 ? launch_rows<Bf16, true>(p, stream, per_round)
+                        : launch_rows<F32, true>(p, stream, per_round);
+    else e = bf16 ? launch_rows<Bf16, false>(p, stream, per_round)
+                  : launch_rows<F32, false>(p, stream, per_round);
   }
   if (e != cudaSuccess) {
     snprintf(err, err_len, "scoring launch failed: %s", cudaGetErrorString(e));

@@ -54,6 +54,7 @@ static int score_case(void) {
   CUDA(cudaMalloc(&d_lx, (size_t)B * V * sizeof(float)));
   CUDA(cudaMalloc(&d_ls, (size_t)B * V * sizeof(float)));
   CUDA(cudaMalloc(&d_ws, ws));
+  CUDA(cudaMemset(d_ws, 0, ws)); /* zero before the first use */
   CUDA(cudaMalloc((void**)&d_state_in, B));
   CUDA(cudaMalloc((void**)&d_state_out, B));
   CUDA(cudaMalloc((void**)&d_conf, B * sizeof(float)));

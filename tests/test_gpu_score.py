@@ -12,6 +12,15 @@ from . import parity as P
 pytestmark = pytest.mark.gpu
 
 
+@pytest.fixture(autouse=True, params=["passes", "fused"])
+def score_path(request, monkeypatch):
+    """Every scoring test runs on both launch paths: the two PDL-chained passes (the
+    default) and the one launch whose M rows wait for their block's C rows (used when the
+    whole grid fits on the device at once; the passes otherwise)."""
+    monkeypatch.setenv("DARD_SCORE_PATH", request.param)
+    return request.param
+
+
 def _run(wl, state_in=None, reps=1, pitch=None):
     ds = DeviceStep(wl, attention=False, logit_pitch=pitch)
     for _ in range(reps):
