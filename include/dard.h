@@ -144,13 +144,35 @@ dard_status dard_step_attention(const dard_attn_args* args, void* stream /* cuda
 
 /* The attention kernel dard_step_attention would launch for these arguments, without
  * launching anything: *kernel = 1 or 2 (the tensor-core kernel with one or two 128-row
- * query tiles per CTA, as the cost model or DARD_ATTN_TC picks), 3 (the fp32 CUDA-core
- * kernel), or 0 (no query rows, no launch). The arguments go through the same host
+ * query tiles per CTA, as the cost model or DARD_ATTN_TC picks), 4 (the kernel on CTA
+ * pairs, head_dim 128, chosen only by DARD_ATTN_TC=4), 3 (the fp32 CUDA-core kernel), or 0
+ * (no query rows, no launch). The arguments go through the same host
  * validation as dard_step_attention and fail with the same codes; device pointers are
  * checked but never read. The cost model uses the current device's SM count (148 when no
  * device is visible, so that the choice can be planned on a host without one). An
  * interface addition: the paper has no counterpart. */
 dard_status dard_attention_kernel(const dard_attn_args* args, int32_t* kernel);
+
+/* The launch plan of dard_step_attention for these arguments, computed on the host without
+ * launching anything (an interface addition: the paper has no counterpart). The arguments
+ * go through the same host validation as dard_step_attention and fail with the same codes.
+ *   kernel              as dard_attention_kernel (0: no query rows, nothing launched)
+ *   ctas                CTAs of the launch (the CTA-pair kernel: two per cluster, as many
+ *                       clusters as fit on the current device, or SMs / 2 without one)
+ *   tile_pairs          (query tile, key tile) pairs a tensor-core kernel computes: 128 query
+ *                       rows of one head against 128 key rows, over every head and sequence
+ *   tile_pairs_skipped  pairs it leaves out because no query of the rows a CTA (or CTA pair)
+ *                       handles attends any key of the tile: tiles holding only shadow keys,
+ *                       for rows that are all original queries of positions after the block
+ *                       (Sec. 3.2, query block 1 attends x copies only). The fp32 kernel,
+ *                       which masks key by key, reports 0 for both.                         */
+typedef struct {
+  int32_t kernel;
+  int64_t ctas;
+  int64_t tile_pairs;
+  int64_t tile_pairs_skipped;
+} dard_attn_plan;
+dard_status dard_attention_plan(const dard_attn_args* args, dard_attn_plan* plan);
 
 /* ------------------------------------------------------------------------------------- *
  * Confidence scoring and state transition (Eq. 1, Eq. 5-8, Algorithm 1).
@@ -249,8 +271,10 @@ dard_status dard_score_and_transition(const dard_score_args* args, void* stream)
  * call depends on what an earlier one left.
  *
  * The first call on each device (the device current at the call) looks up the array's
- * address there once (cudaGetSymbolAddress) and caches it; make that first call before any
- * stream capture on that device. A failed lookup returns DARD_ERR_CUDA.
+ * address there (cudaGetSymbolAddress) and caches it with the current context; a later call
+ * in another context of the device (after a device reset, say) looks it up again. Make the
+ * first call in a context before any stream capture there. A failed lookup returns
+ * DARD_ERR_CUDA.
  *
  * There is one array per device, shared by every call on it: calls whose kernels can
  * overlap on one device (different streams, different host threads) race on it and may

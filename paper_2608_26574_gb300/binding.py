@@ -61,8 +61,14 @@ class DardError(RuntimeError):
 
 _lib = None
 
+class AttnPlan(ctypes.Structure):
+    _fields_ = [("kernel", ctypes.c_int32), ("ctas", ctypes.c_int64),
+                ("tile_pairs", ctypes.c_int64), ("tile_pairs_skipped", ctypes.c_int64)]
+
+
 # Exported entry points: name -> (restype, argtypes)
 EXPORTS = {
+    "dard_attention_plan": (ctypes.c_int, [ctypes.POINTER(AttnArgs), ctypes.POINTER(AttnPlan)]),
     "dard_step_attention": (ctypes.c_int, [ctypes.POINTER(AttnArgs), ctypes.c_void_p]),
     "dard_attention_kernel": (ctypes.c_int, [ctypes.POINTER(AttnArgs),
                                              ctypes.POINTER(ctypes.c_int32)]),
@@ -215,12 +221,22 @@ class AttentionCall:
 
     def kernel(self, q, k, v, o) -> int:
         """The kernel a call on these tensors launches, without launching it: 1 or 2 (the
-        tensor-core kernel with one or two query tiles per CTA), 3 (fp32 CUDA cores), 0 (no
-        query rows)."""
+        tensor-core kernel with one or two query tiles per CTA), 4 (the CTA-pair kernel),
+        3 (fp32 CUDA cores), 0 (no query rows)."""
         self._bind(q, k, v, o)
         out = ctypes.c_int32(-1)
         _check(lib().dard_attention_kernel(self._ref, ctypes.byref(out)), "dard_attention_kernel")
         return int(out.value)
+
+    def plan(self, q, k, v, o) -> dict:
+        """The launch plan of a call on these tensors, without launching it: the kernel, its
+        CTAs, and the (query tile, key tile) pairs it computes and skips."""
+        self._bind(q, k, v, o)
+        out = AttnPlan()
+        _check(lib().dard_attention_plan(self._ref, ctypes.byref(out)), "dard_attention_plan")
+        return {"kernel": int(out.kernel), "ctas": int(out.ctas),
+                "tile_pairs": int(out.tile_pairs),
+                "tile_pairs_skipped": int(out.tile_pairs_skipped)}
 
     def _bind(self, q, k, v, o) -> int:
         """Checks q, k, v and o against the metadata and sets their pointers; returns the

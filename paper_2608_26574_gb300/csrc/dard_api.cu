@@ -247,6 +247,40 @@ dard_status dard_attention_kernel(const dard_attn_args* a, int32_t* kernel) {
   return DARD_OK;
 }
 
+dard_status dard_attention_plan(const dard_attn_args* a, dard_attn_plan* plan) {
+  using namespace dard;
+  g_err[0] = '\0';
+  if (!plan) return fail(DARD_ERR_NULL, "plan is NULL");
+  AttnParams p;
+  const dard_status st = prepare_attention(a, p);
+  if (st != DARD_OK) return st;
+  memset(plan, 0, sizeof(*plan));
+  if (p.total_work == 0) return DARD_OK;
+  plan->kernel = attention_kernel_choice(*a, p);
+  if (plan->kernel == 3) {
+    plan->ctas = p.total_work;
+    return DARD_OK;
+  }
+  plan->ctas = plan->kernel == 1 ? p.total_work
+             : plan->kernel == 2 ? p.total_pairs
+                                 : 2ll * pair_clusters_for(p);
+  // rows handled together: one query tile (kernel 1), or two (kernels 2 and 4)
+  const int unit = plan->kernel == 1 ? kKeyTile : 2 * kKeyTile;
+  for (int s = 0; s < p.num_seqs; ++s) {
+    const SeqDesc& sd = p.seq[s];
+    const int rows = sd.n_orig + sd.slen;
+    const long long all_kt = (rows + kKeyTile - 1) / kKeyTile;
+    for (int r0 = sd.q_start; r0 < rows; r0 += unit) {
+      const int r1 = std::min(r0 + unit, rows);
+      const long long qtiles = (r1 - r0 + kKeyTile - 1) / kKeyTile;
+      const long long used = key_tiles(sd, r0, r1);
+      plan->tile_pairs += qtiles * used * p.hq;
+      plan->tile_pairs_skipped += qtiles * (all_kt - used) * p.hq;
+    }
+  }
+  return DARD_OK;
+}
+
 size_t dard_score_workspace_size(int32_t rows, int32_t vocab, int32_t num_seqs) {
   if (rows < 0 || vocab < 1 || num_seqs < 1 || num_seqs > DARD_MAX_SEQS) return 0;
   return dard::score_workspace_bytes(rows, num_seqs);

@@ -113,8 +113,8 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
   decode_work(p, blockIdx.x, seq, qt, h);
   const SeqDesc sd = p.seq[seq];
   const int rows_seq = sd.n_orig + sd.slen;
-  const int n_kt = (rows_seq + kTN - 1) / kTN;
   const int q0 = sd.q_start + qt * kBM;  // first (sequence-relative) query row of the tile
+  const int n_kt = key_tiles(sd, q0, min(q0 + kBM, rows_seq));  // shadow-only tiles skipped
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -564,9 +564,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   decode_pair(p, blockIdx.x, seq, pr, h);
   const SeqDesc sd = p.seq[seq];
   const int rows_seq = sd.n_orig + sd.slen;
-  const int n_kt = (rows_seq + kTN - 1) / kTN;
   const int qt0 = kQT * pr;                       // first query tile of this CTA
   const int nq = min(kQT, sd.n_qtiles - qt0);     // 1 or 2 query tiles
+  const int r0 = sd.q_start + qt0 * kBM;
+  const int n_kt = key_tiles(sd, r0, min(r0 + nq * kBM, rows_seq));  // shadow-only tiles skipped
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row0 = sd.row_base;
@@ -994,6 +995,16 @@ dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_
                              char* err, size_t err_len) {
   cudaError_t e;
   const int kernel = attention_kernel_choice(a, p);
+  // Test hooks (failure-path tests; unset in normal operation): a bound on every in-kernel
+  // wait, a K copy the pair kernel never issues (its waits then run out), a launch that
+  // reports failure without launching.
+  if (const char* w = std::getenv("DARD_TEST_WAIT_CYCLES")) p.wait_cycles = std::atoll(w);
+  if (const char* d = std::getenv("DARD_TEST_DROP_KV")) p.test_drop_kv = std::atoi(d);
+  if (std::getenv("DARD_TEST_FAIL_LAUNCH") != nullptr) {
+    snprintf(err, err_len, "attention launch failed: %s (DARD_TEST_FAIL_LAUNCH)",
+             cudaGetErrorString(cudaErrorLaunchFailure));
+    return DARD_ERR_CUDA;
+  }
   if (kernel == 3) {
     if (a.head_dim == 64) attn_simt<64><<<p.total_work, 256, 0, stream>>>(p);
     else attn_simt<128><<<p.total_work, 256, 0, stream>>>(p);

@@ -190,8 +190,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       int use = 0;
-      int last_use[kPST];
-      for (int b = 0; b < kPST; ++b) last_use[b] = -1;
+      int k_last[kPST], v_last[kPST];  // the latest use of each stage whose copy was issued
+      for (int b = 0; b < kPST; ++b) k_last[b] = v_last[b] = -1;
       bool ok = true;
       for (int w = cid; w < p.total_pairs && ok; w += ncl) {
         const PairItem it = pair_item(p, w);
@@ -210,25 +210,26 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           ok = !*abort_flag && (use < kPST || mbar_wait(&ctl.k_empty[b], ph, wlim));
           if (!ok) break;
           mbar_arrive_expect_tx(&ctl.k_land[b], kHalf);
-          if (use != p.test_drop_kv) {  // test hook: a dropped copy never lands
+          if (use != p.test_drop_kv) {  // test hook: a dropped copy is never issued
             tma_load_2d(sK + b * kHalf, &tmk, &ctl.k_land[b], kc, row0 + j * kTN + 64 * rank);
             tma_load_2d(sK + b * kHalf + kKBlock, &tmk, &ctl.k_land[b], kc + 64,
                         row0 + j * kTN + 64 * rank);
+            k_last[b] = use;
           }
           ok = use < kPST || mbar_wait(&ctl.v_empty[b], ph, wlim);
           if (!ok) break;
           mbar_arrive_expect_tx(&ctl.v_land[b], kHalf);
           tma_load_2d(sV + b * kHalf, &tmv, &ctl.v_land[b], kc + 64 * rank, row0 + j * kTN);
-          last_use[b] = use;
+          v_last[b] = use;
         }
       }
       if (!ok) pair_flag_timeout(p, ctl);
-      // Own copies in flight land before shared memory is released (bounded: a copy that
-      // was never issued, or never lands, gives up).
+      // Every copy this CTA issued lands before shared memory is released: the latest
+      // issued use of each stage (earlier uses of a stage landed before it was reused).
       for (int b = 0; b < kPST; ++b) {
-        if (last_use[b] < 0) continue;
-        const uint32_t ph = (last_use[b] / kPST) & 1;
-        if (!mbar_wait(&ctl.k_land[b], ph, wlim) || !mbar_wait(&ctl.v_land[b], ph, wlim))
+        if (k_last[b] >= 0 && !mbar_wait(&ctl.k_land[b], (k_last[b] / kPST) & 1, wlim))
+          pair_flag_timeout(p, ctl);
+        if (v_last[b] >= 0 && !mbar_wait(&ctl.v_land[b], (v_last[b] / kPST) & 1, wlim))
           pair_flag_timeout(p, ctl);
       }
     }
@@ -330,9 +331,11 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     // Thread 0: the Q tile of an item (this CTA's 128 rows, two 64-column swizzled blocks)
     // by TMA into the staging buffer, which is free (every softmax thread has passed the
     // barrier after its last use).
-    int q_loads = 0;  // Q tiles taken out of the staging buffer so far (q_land phases)
+    int q_loads = 0;   // Q tiles taken out of the staging buffer so far (q_land phases)
+    int q_issued = 0;  // Q tile loads issued (thread 0)
     auto load_q = [&](const PairItem& qi) {
       if (threadIdx.x == 0) {
+        ++q_issued;
         const int row = p.seq[qi.seq].row_base + qi.r0 + kBM * static_cast<int>(rank);
         fence_proxy_async_smem();  // the buffer's generic reads and writes come first
         mbar_arrive_expect_tx(&ctl.q_land, 2 * kHalf);
@@ -546,6 +549,11 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       if (w + 2 * ncl < p.total_pairs) load_q(pair_item(p, w + 2 * ncl));
       it = pair_item(p, w + ncl);
     }
+    // A Q tile load issued but not taken out (an item left early) lands before shared
+    // memory is released; at most the latest one is outstanding.
+    if (threadIdx.x == 0 && q_issued > q_loads &&
+        !mbar_wait(&ctl.q_land, (q_issued - 1) & 1, wlim))
+      pair_flag_timeout(p, ctl);
   }
   // ------------------------------------------------------------ teardown
   __syncwarp();
@@ -581,7 +589,7 @@ int pair_max_clusters(size_t smem) {
   cfg.numAttrs = 1;
   if (cudaOccupancyMaxActiveClusters(&n, attn_pair, &cfg) != cudaSuccess || n <= 0) {
     cudaGetLastError();
-    n = sm_count() / 2;
+    return sm_count() / 2;  // not cached: the query may succeed once the attributes are set
   }
   cache[dev].store(n, std::memory_order_relaxed);
   return n;

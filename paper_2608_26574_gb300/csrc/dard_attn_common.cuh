@@ -277,14 +277,7 @@ __device__ RowMasks row_masks(const RowInfo& q, const BlockInfo& bi, const SeqDe
 constexpr int kTN = 128;  // keys per tile of the tensor-core path
 constexpr int kL2Ahead = 4;  // K/V tiles prefetched into L2 ahead of the TMA loads
 
-// Key tiles that query rows [r0, r1) of a sequence need. Original queries of positions after
-// the block (query block 1 of Sec. 3.2: M positions attend the x copy of every position) never
-// see a shadow key, so a run of such rows stops before the tiles that hold shadow keys only;
-// every other run of rows needs all tiles of the sequence.
-__host__ __device__ inline int key_tiles(const SeqDesc& sd, int r0, int r1) {
-  if (r0 >= sd.b0 + sd.blen && r1 <= sd.n_orig) return (sd.n_orig + kTN - 1) / kTN;
-  return (sd.n_orig + sd.slen + kTN - 1) / kTN;
-}
+static_assert(kTN == kKeyTile, "one key-tile width for the kernels and the planner");
 
 __device__ __forceinline__ bool tile_needs_mask(const SeqDesc& sd, int kt0) {
   return (kt0 + kTN > sd.n_orig) ||

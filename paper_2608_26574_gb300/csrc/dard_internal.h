@@ -24,6 +24,18 @@ struct SeqDesc {
   int32_t n_qtiles;   // ceil((N + S - q_start) / 128)
 };
 
+// Keys per tile of the tensor-core attention kernels.
+constexpr int kKeyTile = 128;
+
+// Key tiles that query rows [r0, r1) of a sequence need. Original queries of positions after
+// the block (query block 1 of Sec. 3.2: M positions attend the x copy of every position) never
+// see a shadow key, so a run of such rows stops before the tiles that hold shadow keys only;
+// every other run of rows needs all tiles of the sequence.
+__host__ __device__ inline int key_tiles(const SeqDesc& sd, int r0, int r1) {
+  if (r0 >= sd.b0 + sd.blen && r1 <= sd.n_orig) return (sd.n_orig + kKeyTile - 1) / kKeyTile;
+  return (sd.n_orig + sd.slen + kKeyTile - 1) / kKeyTile;
+}
+
 struct AttnParams {
   const uint8_t* state;
   const float* prev_conf;

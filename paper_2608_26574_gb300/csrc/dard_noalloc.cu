@@ -6,7 +6,8 @@
 // state). Here it is a file-scope __device__ array sized for DARD_SCORE_NOALLOC_MAX_ROWS
 // rows and DARD_MAX_SEQS sequences. Its address on a device is looked up once
 // (cudaGetSymbolAddress, with that device current) on the first call made on that device,
-// cached per device, and then passed as the workspace of dard_score_and_transition, whose
+// cached per device together with the context it belongs to (looked up again when the
+// current context changes), and then passed as the workspace of dard_score_and_transition, whose
 // kernels and validation run unchanged. Every call first clears the counters with an
 // asynchronous memset on its stream, so a call never depends on what an earlier one left
 // behind. No call allocates or frees device memory.
@@ -26,20 +27,46 @@ __device__ __align__(256) uint8_t g_score_scratch[kScratchBytes];
 constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
 void* g_scratch_ptr[kMaxDevices] = {};
+void* g_scratch_ctx[kMaxDevices] = {};  // the context the cached address belongs to
 
-// Device address of g_score_scratch on the current device (looked up on first use).
+// The current CUDA context (driver entry point, so that the library needs no -lcuda).
+cudaError_t current_context(void** ctx) {
+  using GetCurrent = int (*)(void**);
+  static GetCurrent fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<GetCurrent>(f);
+  });
+  if (fn == nullptr) return cudaErrorNotSupported;
+  return fn(ctx) == 0 ? cudaSuccess : cudaErrorUnknown;
+}
+
+// Device address of g_score_scratch on the current device: looked up on the first call in
+// a context, and again whenever the current context has changed (a device reset or a new
+// primary context loads the module again, at another address).
 cudaError_t scratch_on_current_device(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  void* ctx = nullptr;
+  e = current_context(&ctx);  // NULL before the runtime has initialised the device
+  if (e != cudaSuccess) return e;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (g_scratch_ptr[dev] == nullptr) {
+  if (g_scratch_ptr[dev] == nullptr || ctx == nullptr || g_scratch_ctx[dev] != ctx) {
     void* ptr = nullptr;
-    e = cudaGetSymbolAddress(&ptr, g_score_scratch);
+    e = cudaGetSymbolAddress(&ptr, g_score_scratch);  // initialises the context if needed
     if (e != cudaSuccess) return e;
     if (ptr == nullptr) return cudaErrorInvalidSymbol;
+    e = current_context(&ctx);
+    if (e != cudaSuccess) return e;
     g_scratch_ptr[dev] = ptr;
+    g_scratch_ctx[dev] = ctx;
   }
   *out = g_scratch_ptr[dev];
   return cudaSuccess;

@@ -955,6 +955,13 @@ dard_status launch_score(const dard_score_args& a, ScoreParams& p, cudaStream_t 
   p.new_state = p.pd_flag + align256(static_cast<size_t>(p.rows));
   p.log2_lambda = static_cast<float>(std::log2(static_cast<double>(p.lambda)));
 
+  // Test hook (failure-path tests; unset in normal operation): a launch that reports
+  // failure without launching.
+  if (std::getenv("DARD_TEST_FAIL_LAUNCH") != nullptr) {
+    snprintf(err, err_len, "scoring launch failed: %s (DARD_TEST_FAIL_LAUNCH)",
+             cudaGetErrorString(cudaErrorLaunchFailure));
+    return DARD_ERR_CUDA;
+  }
   cudaError_t e = cudaSuccess;
   if (p.counts != nullptr && p.rows == 0) {
     zero_all_counts<<<1, 256, 0, stream>>>(p);

@@ -173,3 +173,55 @@ def test_binding_raises_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(B, "_lib", None)
     with pytest.raises(RuntimeError, match="missing"):
         B.lib(str(tmp_path / "libdard.so"))
+
+
+def _plan(lib, **kw):
+    a, keep = _attn_args(**kw)
+    out = B.AttnPlan()
+    assert lib.dard_attention_plan(ctypes.byref(a), ctypes.byref(out)) == 0
+    return out
+
+
+@pytest.mark.parametrize("tc", ["1", "2", "4"])
+def test_attention_plan_counts_skipped_tile_pairs(lib, monkeypatch, tc):
+    """The host-only plan counts the (query tile, key tile) pairs each tensor-core kernel
+    computes and skips: a key tile holding only shadow rows is skipped for the rows a CTA
+    (or CTA pair) handles when they are all original queries of positions after the block
+    (Sec. 3.2, query block 1 attends x copies only). Expected counts are worked out from the
+    layout of each case by hand."""
+    monkeypatch.setenv("DARD_ATTN_TC", tc)
+    i32 = lambda *x: np.array(x, np.int32)  # noqa: E731
+    # 8B layer: 768 original rows, block [608, 640), 32 shadow rows -> 800 rows, 7 key tiles;
+    # 7 query tiles per head. Query tile 5 (rows 640..767) is all future-block rows.
+    p = _plan(lib, n=i32(768), b0=i32(608), bl=i32(32), sl=i32(32), hq=32, hkv=32,
+              head_dim=128)
+    assert p.kernel == int(tc)
+    assert p.tile_pairs + p.tile_pairs_skipped == 7 * 7 * 32
+    # one-tile units: tile 5 skips key tile 6; 256-row units [512, 768) hold prompt rows
+    assert p.tile_pairs_skipped == (32 if tc == "1" else 0)
+    # GQA layer: 5120 original rows, block [4608, 4672), 64 shadow rows -> 5184 rows, 41 key
+    # tiles, 41 query tiles per head; rows 4672..5119 are future-block rows.
+    p = _plan(lib, n=i32(5120), b0=i32(4608), bl=i32(64), sl=i32(64), hq=28, hkv=4,
+              head_dim=128)
+    assert p.tile_pairs + p.tile_pairs_skipped == 41 * 41 * 28
+    # one-tile units 37, 38, 39 (rows 4736..5119); two-tile unit [4864, 5120) = 2 tiles
+    assert p.tile_pairs_skipped == (3 * 28 if tc == "1" else 2 * 28)
+    # no shadow rows: nothing to skip
+    p = _plan(lib, n=i32(300), b0=i32(100), bl=i32(32), sl=i32(0), hq=4, hkv=4, head_dim=128)
+    assert p.tile_pairs_skipped == 0 and p.tile_pairs == 3 * 3 * 4
+
+
+def test_attention_plan_fp32_and_empty(lib, monkeypatch):
+    monkeypatch.delenv("DARD_ATTN_TC", raising=False)
+    p = _plan(lib, dtype=B.DARD_F32)
+    assert p.kernel == 3 and p.ctas >= 1 and p.tile_pairs == 0 and p.tile_pairs_skipped == 0
+    p = _plan(lib, qs=np.array([96], np.int32))  # every row before query_start: no launch
+    assert p.kernel == 0 and p.ctas == 0 and p.tile_pairs == 0
+
+
+def test_attention_plan_validates_like_the_launch(lib):
+    a, keep = _attn_args(head_dim=96)
+    out = B.AttnPlan()
+    assert lib.dard_attention_plan(ctypes.byref(a), ctypes.byref(out)) == 4
+    assert lib.dard_attention_plan(ctypes.byref(a), None) == 1
+    assert lib.dard_attention_plan(None, ctypes.byref(out)) == 1

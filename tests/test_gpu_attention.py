@@ -297,3 +297,29 @@ def test_attention_no_query_rows(tc):
     ds.attention(0, out=out)
     torch.cuda.synchronize()
     assert bool((out == 7.0).all())
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_mask_probe_skipped_shadow_tiles(d, tc):
+    """Long runs of rows after the block (original queries of M positions attend x copies
+    only, Sec. 3.2 query block 1): their CTAs skip the key tiles that hold only shadow rows.
+    Uniform attention (Q = 0) shows that nothing they should see was skipped, and the host
+    plan reports the skipped pairs."""
+    specs = [dict(n_orig=700, block_start=100, block_len=64, fractions=(0.3, 0.4, 0.3)),
+             dict(n_orig=900, block_start=0, block_len=128, fractions=(0.4, 0.3, 0.3)),
+             dict(n_orig=640, block_start=200, block_len=32, fractions=(0.2, 0.5, 0.3),
+                  shadow="candidates")]
+    wl = W.custom(specs, 4, 2, d, probe=True, seed=31 + d)
+    ds = DeviceStep(wl, layers=[0], scoring=False)
+    q, k, v, o = ds.layers[0]
+    plan = ds.attention_call().plan(q, k, v, o)
+    assert plan["tile_pairs_skipped"] > 0, plan
+    o = ds.attention(0).float().cpu().numpy()
+    torch.cuda.synchronize()
+    mx, mean, n = P.compare_attention(wl, 0, o)
+    # a wrongly skipped tile drops up to 64 attended keys of ~700 and moves a row's mean of
+    # N(0, 1) values by ~1e-2; the bf16 output rounding stays within half an ulp of |O|
+    tol = max(_probe_tol(wl), 3 * 2.0 ** -9 * float(abs(o).max()))
+    print("skip probe", d, plan, mx, mean, n, tol)
+    assert mx <= tol
+    assert int(ds.status.item()) == 0
