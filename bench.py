@@ -15,6 +15,10 @@ results inside the timed region, two steps in flight (step i + 1's inputs cross 
 link, ~0.2 TB/s and the bound of this number, while step i computes); the one-step-at-a-time
 figure is reported beside it.
 
+Per-config block: attention (and its prefix-cached variant) and scoring of every workload
+(tiny, 8B, GQA, ragged, multimodal; the multimodal one also as its 32-layer step), CUDA-graph
+timing over rotating device input sets drawn with each workload's distributions.
+
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 """
 from __future__ import annotations
@@ -53,6 +57,9 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-per-config", action="store_true")
+    ap.add_argument("--soak-seconds", type=float, default=2.5)
+    ap.add_argument("--oracle-one-core", action="store_true", help=argparse.SUPPRESS)
     return ap.parse_args()
 
 
@@ -183,6 +190,196 @@ def cpu_baseline(wl, seconds: float) -> dict:
                       f"threads, the rest of numpy on 1"}
 
 
+# ------------------------------------------------------------------------------ per-config timing
+def device_bulk(wl, dev, seed, layers=1, logits=True):
+    """Seeded device tensors drawn with the workload's distributions: Q/K/V per layer (each
+    row's own std), and the two logit tensors (N(0, std) with the planted peaks). Timing
+    inputs only: no timed quantity depends on the values."""
+    import torch
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    rows = wl.total_rows
+    std = torch.tensor(wl.row_std, dtype=torch.float32, device=dev)[:, None, None]
+    qkv = []
+    for _ in range(layers):
+        qkv.append(tuple((torch.randn(rows, h, wl.head_dim, generator=g, device=dev) * std).to(dt)
+                         for h in (wl.hq, wl.hkv, wl.hkv)))
+    lg = None
+    if logits:
+        lstd, frac, height = wl.logit_spec
+        nrows = wl.total_block
+        lg = []
+        for _ in range(2):
+            t = torch.randn(nrows, wl.vocab, generator=g, device=dev) * lstd
+            n_plant = int(round(frac * nrows))
+            if n_plant:
+                r = torch.randperm(nrows, generator=g, device=dev)[:n_plant]
+                c = torch.randint(0, wl.vocab, (n_plant,), generator=g, device=dev)
+                t[r, c] += height
+            lg.append(t.to(dt))
+    return qkv, lg
+
+
+def graph_us(calls, min_seconds=0.15):
+    """Average microseconds per call: a CUDA graph of `calls` (one per rotating input set),
+    replayed back to back between CUDA events for about `min_seconds`."""
+    import torch
+    for c in calls:
+        c()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for c in calls:
+            c()
+    g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    g.replay()
+    e1.record()
+    e1.synchronize()
+    once = max(e0.elapsed_time(e1) * 1e-3, 1e-6)
+    reps = max(3, int(min_seconds / once))
+    e0.record()
+    for _ in range(reps):
+        g.replay()
+    e1.record()
+    e1.synchronize()
+    return e0.elapsed_time(e1) * 1e3 / (reps * len(calls))
+
+
+def n_sets(bytes_per_set, floor=2, cap=16, target=600e6):
+    """Input sets for rotation: together more than 4x the 129 MB L2 (or at least `floor`)."""
+    return int(max(floor, min(cap, math.ceil(target / max(bytes_per_set, 1)))))
+
+
+def per_config(dev, hbm, bf16):
+    """Attention and scoring of every workload (and the prefix-cached variants), CUDA-graph
+    timing over rotating device input sets; the multimodal config also as its 32-layer
+    step (32 attention launches and one scoring call)."""
+    import numpy as np
+    import torch
+    from paper_2608_26574_gb300 import binding as Bd
+    from paper_2608_26574_gb300 import workloads as W
+    from paper_2608_26574_gb300.device import DeviceStep
+    kernels = {1: "attn_tc1", 2: "attn_tc2", 3: "attn_simt", 4: "attn_pair"}
+    out = {}
+    for name in ("tiny", "8b", "gqa", "ragged", "mm"):
+        entry = {}
+        for prefix in (False, True):
+            wl = W.make(name, attention=False, scoring=False, prefix=prefix)
+            meta = DeviceStep(wl, device=dev, attention=False, scoring=False)
+            call = meta.attention_call()
+            per = wl.total_rows * (wl.hq + 2 * wl.hkv) * wl.head_dim * (2 if wl.dtype == "bf16" else 4)
+            ns = n_sets(per)
+            qkv, _ = device_bulk(wl, dev, 5000 + W.CONFIG_INDEX[name], layers=ns, logits=False)
+            outs = [torch.empty_like(q) for q, _, _ in qkv]
+            plan = call.plan(qkv[0][0], qkv[0][1], qkv[0][2], outs[0])
+            us = graph_us([lambda i=i: call(*qkv[i], outs[i]) for i in range(ns)])
+            flops = W.attention_flops(wl)
+            tf = flops / (us * 1e-6) / 1e12
+            rec = {"us": us, "tflops": tf, "frac_bf16": tf / bf16 if wl.dtype == "bf16" else None,
+                   "kernel": kernels.get(plan["kernel"], str(plan["kernel"])),
+                   "gflop": flops / 1e9, "tile_pairs": plan["tile_pairs"],
+                   "tile_pairs_skipped": plan["tile_pairs_skipped"], "input_sets": ns}
+            entry["attention_prefix" if prefix else "attention"] = rec
+            if name == "mm" and not prefix:
+                # the multimodal step: 32 layers of attention and the block's scoring
+                wls = W.make(name, attention=False, scoring=False)
+                _, lg = device_bulk(wls, dev, 6000, layers=0)
+                sc = _score_call(wls, meta, dev)
+                layer_calls = [lambda i=i: call(*qkv[i % ns], outs[i % ns]) for i in range(32)]
+                step = layer_calls + [lambda: sc(lg[0], lg[1])]
+                us_step = graph_us(step, min_seconds=0.3) * len(step)
+                entry["step_32_layers"] = {"us": us_step, "layers": 32,
+                                           "attention_tflops": 32 * flops / (us_step * 1e-6) / 1e12}
+            del qkv, outs
+            torch.cuda.empty_cache()
+        wl = W.make(name, attention=False, scoring=False)
+        meta = DeviceStep(wl, device=dev, attention=False, scoring=False)
+        esz = 2 if wl.dtype == "bf16" else 4
+        ns = n_sets(2 * wl.total_block * wl.vocab * esz)
+        lgs = [device_bulk(wl, dev, 7000 + k, layers=0)[1] for k in range(ns)]
+        sc = _score_call(wl, meta, dev)
+        us = graph_us([lambda i=i: sc(lgs[i][0], lgs[i][1]) for i in range(ns)])
+        by = W.scoring_bytes(wl)
+        gbs = by / (us * 1e-6) / 1e9
+        entry["scoring"] = {"us": us, "gbs": gbs, "frac_hbm": gbs / hbm, "frac_8tbs": gbs / 8000.0,
+                            "bytes": by, "rows": wl.total_block, "input_sets": ns}
+        entry["status_word"] = int(meta.status.item())
+        out[name] = entry
+        del lgs
+        torch.cuda.empty_cache()
+    return out
+
+
+def _score_call(wl, meta, dev):
+    """A prepared scoring call over fresh output buffers and a zeroed workspace."""
+    import torch
+    from paper_2608_26574_gb300 import binding as Bd
+    r = max(wl.total_block, 1)
+    ws = torch.zeros(max(Bd.dard_score_workspace_size(wl.total_block, wl.vocab, len(wl.seqs)), 16),
+                     dtype=torch.uint8, device=dev)
+    bufs = dict(conf=torch.empty(r, dtype=torch.float32, device=dev),
+                token=torch.empty(r, dtype=torch.int32, device=dev),
+                state_out=torch.empty(r, dtype=torch.uint8, device=dev),
+                w_out=torch.empty(r, dtype=torch.float32, device=dev),
+                counts=torch.empty(3 * len(wl.seqs), dtype=torch.int32, device=dev))
+    call = Bd.ScoreCall(meta.block_len, meta.state, wl.tau_c, wl.tau_u, wl.lam, wl.p0,
+                        bufs["conf"], bufs["token"], bufs["state_out"], ws, w_out=bufs["w_out"],
+                        counts=bufs["counts"], status=meta.status)
+    call._keep_bufs = (bufs, ws)
+    return call
+
+
+def cpu_one_core(seconds: float) -> dict | None:
+    """The oracle on one host core: a child process with every BLAS pool at one thread, on a
+    sample of the 8B step's query rows (all heads) and its scoring block, extrapolated to a
+    full step by rows."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    try:
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-one-core",
+                            "--cpu-seconds", str(seconds)], env=env, capture_output=True,
+                           text=True, timeout=seconds * 6 + 60)
+        return json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception as e:  # noqa: BLE001 - the figure is optional
+        return {"error": str(e)[:200]}
+
+
+def oracle_one_core(seconds: float):
+    """Child of cpu_one_core: time the oracle and print one JSON line."""
+    import numpy as np
+    from paper_2608_26574_gb300 import workloads as W
+    import oracle as orc
+    wl = W.make("8b")
+    s = wl.seqs[0]
+    lay = orc.SeqLayout(s.n_orig, s.block_start, s.state, s.prev_conf, s.shadow_src)
+    rows_total = s.rows
+    a_t, a_rows, sc_t, sc_n, cursor = 0.0, 0, 0.0, 0, 0
+    t_end = time.perf_counter() + seconds
+    while time.perf_counter() < t_end or sc_n == 0:
+        rows = (cursor + np.arange(32)) % rows_total
+        cursor = (cursor + 32) % rows_total
+        t0 = time.perf_counter()
+        mask = orc.attention_mask(lay, rows=rows)
+        orc.masked_attention(wl.q[0], wl.k[0], wl.v[0], mask, rows=rows)
+        a_t += time.perf_counter() - t0
+        a_rows += len(rows)
+        if sc_n == 0 or a_rows % 256 == 0:
+            t1 = time.perf_counter()
+            orc.score_block(wl.logits_x, wl.logits_s, s.state, float(np.float32(wl.tau_c)),
+                            float(np.float32(wl.tau_u)), float(np.float32(wl.lam)),
+                            float(np.float32(wl.p0)))
+            sc_t += time.perf_counter() - t1
+            sc_n += 1
+    per = (a_t / a_rows * rows_total + sc_t / sc_n) * 1e6
+    print(json.dumps({"value": per, "unit": "µs", "cores": 1, "kind": "oracle",
+                      "sample": f"{a_rows} query-row evaluations (rows taken in turn from the 8B step's {rows_total}; all 32 heads) "
+                                f"and {sc_n} scoring blocks, extrapolated to a full step by rows; "
+                                f"BLAS on 1 thread"}))
+
+
 # ------------------------------------------------------------------------------ reference arm
 def run_reference(args, rank: int):
     if rank != 0:
@@ -305,8 +502,13 @@ def run_ours(args, rank: int, world: int):
         e1.synchronize()
         return e0.elapsed_time(e1)
 
+    # Clocks are sampled (every 100 ms) over a window that holds a soak of back-to-back
+    # step graphs (at least 20 samples, the sustained figure) followed by the timed region
+    # of exactly `steps` steps.
     mon = ClockMonitor(local)
     mon.start()
+    soak_reps = max(1, int(args.soak_seconds / max(timed(g_step, 1) * 1e-3, 1e-6)))
+    soak_ms = timed(g_step, soak_reps)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -317,6 +519,8 @@ def run_ours(args, rank: int, world: int):
     clocks = mon.stop()
     ms = max_over_ranks(ms, world, dev)
     ms_per_step = ms / args.steps
+    sustained = {"ms_per_step": soak_ms / (soak_reps * NSETS), "steps": soak_reps * NSETS,
+                 "seconds": soak_ms * 1e-3}
 
     # per-kernel averages (same launches, one kernel per graph)
     reps = max(4, min(400, int(0.25 / max(ms_per_step / 1e3, 1e-6) / NSETS)))
@@ -442,14 +646,21 @@ def run_ours(args, rank: int, world: int):
                 "serial_value": e2e_serial_us, "results_match_device_step": e2e_ok},
         "gpu_launches": args.steps * 3,
         "status_word": status,
+        "sustained": sustained,
     }
+    if not args.no_per_config:
+        line["per_config"] = per_config(dev, hbm, bf16)
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
+        line["cpu_baseline_one_core"] = cpu_one_core(args.cpu_seconds / 2)
     print(json.dumps(line), flush=True)
 
 
 def main():
     args = parse()
+    if args.oracle_one_core:
+        oracle_one_core(args.cpu_seconds)
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":

@@ -41,12 +41,16 @@ CONFIG_INDEX = {"tiny": 0, "8b": 1, "gqa": 2, "ragged": 3, "mm": 4}
 
 
 def round_bf16(a: np.ndarray) -> np.ndarray:
-    """Round float32 values to the nearest bfloat16 (ties to even); returns float32."""
-    a = np.ascontiguousarray(a, dtype=np.float32)
-    bits = a.view(np.uint32).astype(np.uint64)
-    bias = ((bits >> 16) & 1) + 0x7FFF
-    out = ((bits + bias) & 0xFFFF0000).astype(np.uint32)
-    return out.view(np.float32)
+    """Round float32 values to the nearest bfloat16 (ties to even); returns float32.
+    Finite inputs only: the largest finite pattern plus the rounding bias stays below 2^32,
+    so the sum is formed in uint32."""
+    bits = np.array(a, dtype=np.float32, copy=True).view(np.uint32)
+    bias = bits >> np.uint32(16)
+    bias &= np.uint32(1)
+    bias += np.uint32(0x7FFF)
+    bits += bias
+    bits &= np.uint32(0xFFFF0000)
+    return bits.view(np.float32)
 
 
 def state_counts(B: int, fractions: tuple[float, float, float]) -> list[int]:
@@ -103,6 +107,8 @@ class Workload:
     v: list = field(default_factory=list)
     logits_x: np.ndarray | None = None      # float32 [sum B, vocab]
     logits_s: np.ndarray | None = None
+    row_std: np.ndarray | None = None       # per-row std of Q, K and V
+    logit_spec: tuple | None = None         # logits: (std, planted fraction, planted height)
 
     @property
     def total_rows(self) -> int:
@@ -249,6 +255,9 @@ def make(name: str, layout: str = "paper", logits: str = "literal", attention: b
     if prefix:
         for sq in wl.seqs:
             sq.query_start = sq.prompt
+    # the distributions, for callers that draw the bulk tensors elsewhere (on the device)
+    wl.row_std = np.asarray(std_fn(sum(sq.rows for sq in wl.seqs)), dtype=np.float64)
+    wl.logit_spec = lspec
     if attention:
         for _ in range(wl.layers):
             q, k, v = _qkv(rng, wl.seqs, wl.hq, wl.hkv, wl.head_dim, wl.dtype, std_fn)
