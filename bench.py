@@ -284,6 +284,19 @@ def per_config(dev, hbm, bf16):
                    "gflop": flops / 1e9, "tile_pairs": plan["tile_pairs"],
                    "tile_pairs_skipped": plan["tile_pairs_skipped"], "input_sets": ns}
             entry["attention_prefix" if prefix else "attention"] = rec
+            if not prefix:
+                # the same call with RoPE applied inside it (q, k before RoPE; the key pass
+                # and the attention kernel, chained by programmatic dependent launch)
+                call_r = meta.attention_call(rope=(500000.0, Bd.DARD_ROPE_INTERLEAVED))
+                krs = [torch.empty_like(k) for _, k, _ in qkv]
+                us_r = graph_us([lambda i=i: call_r(*qkv[i], outs[i], k_rope=krs[i])
+                                 for i in range(ns)])
+                tf_r = flops / (us_r * 1e-6) / 1e12
+                entry["attention_rope"] = {
+                    "us": us_r, "tflops": tf_r,
+                    "frac_bf16": tf_r / bf16 if wl.dtype == "bf16" else None,
+                    "rope_us": us_r - us, "theta": 500000.0, "pairing": "interleaved"}
+                del krs
             if name == "mm" and not prefix:
                 # the multimodal step: 32 layers of attention and the block's scoring
                 wls = W.make(name, attention=False, scoring=False)

@@ -130,7 +130,36 @@ typedef struct {
                                 caching: the prompt's outputs are not recomputed, its
                                 K/V rows still serve as keys); rows before q_i of o are
                                 left untouched. NULL means 0 for every sequence.           */
+  /* Rotary position embedding inside the call (Sec. 3.1: x^i and s^i share the positional
+   * embedding of position i). rope_theta = 0: q and k already carry their positions (no
+   * rotation here, k_rope unused). rope_theta >= 1: q and k arrive before RoPE and the call
+   * rotates them, original row r of a sequence at position r and shadow row N_i + k at
+   * position shadow_src[k]; see "RoPE" below. */
+  float rope_theta;          /* 0, or the RoPE base theta >= 1                             */
+  int32_t rope_style;        /* dard_rope_style: which elements form a rotated pair        */
+  void* k_rope;              /* device [total_rows, hkv, head_dim], dtype: receives k after
+                                RoPE, the keys the attention reads (a key cache may take
+                                it); may be k itself (rotated in place). Required when
+                                rope_theta > 0, 16-byte aligned.                           */
 } dard_attn_args;
+
+/* RoPE (rotary position embedding, Su et al., RoFormer, 2021) as dard_step_attention applies
+ * it when rope_theta > 0. For head dimension D and frequency index i in 0 .. D/2 - 1 the
+ * pair (a, b) of a row at position p is replaced by
+ *     (a cos(p f_i) - b sin(p f_i),  a sin(p f_i) + b cos(p f_i)),   f_i = theta^(-2i/D),
+ * in every head of q and of k. DARD_ROPE_INTERLEAVED pairs elements (2i, 2i + 1);
+ * DARD_ROPE_HALF pairs (i, i + D/2). The call first rotates k into k_rope (one pass over the
+ * key rows, launched on the stream ahead of the attention kernel, which waits for it with
+ * programmatic dependent launch), then the attention kernel rotates each query tile as it
+ * loads it; the rotated q is not written out. Arithmetic: the angle p f_i is carried in two
+ * floats (f_i split into a float and its remainder), reduced modulo 2 pi with a two-constant
+ * additive (Cody-Waite) split of 2 pi, and its cosine and sine taken by the hardware
+ * approximations on the reduced angle (absolute error near 1e-6 in all); rotated values are
+ * rounded to dtype. Every N_i must be at most 2^20 (DARD_ERR_SHAPE). A shadow row whose
+ * shadow_src is invalid (DARD_STATUS_BAD_SHADOW) is rotated by an unspecified angle; it is a
+ * masked-out key and an unwritten query row anyway. */
+typedef enum { DARD_ROPE_INTERLEAVED = 0, DARD_ROPE_HALF = 1 } dard_rope_style;
+#define DARD_ROPE_MAX_POSITIONS (1 << 20)
 
 /* Rows are total_rows = sum_i (N_i + S_i). q, k, v, o must be 16-byte aligned; with dtype
  * BF16 a tensor-core kernel runs (head_dim 64 or 128), with F32 the CUDA-core kernel.
@@ -138,8 +167,9 @@ typedef struct {
  * picks the one a cost model of the batch (query tiles, key tiles, SM count) predicts to be
  * faster; the environment variable DARD_ATTN_TC=1 or 2 forces one of them (results agree
  * within rounding).
- * Errors: DARD_ERR_NULL, _SHAPE, _VALUE (scale < 0 or not finite), _UNSUPPORTED,
- * _ALIGN, _CUDA. */
+ * Errors: DARD_ERR_NULL (also: k_rope NULL with rope_theta > 0), _SHAPE, _VALUE (scale < 0
+ * or not finite; rope_theta neither 0 nor a finite value >= 1; rope_style not a
+ * dard_rope_style), _UNSUPPORTED, _ALIGN, _CUDA. */
 dard_status dard_step_attention(const dard_attn_args* args, void* stream /* cudaStream_t */);
 
 /* The attention kernel dard_step_attention would launch for these arguments, without

@@ -9,7 +9,9 @@ Everything is written for a reader to check against the paper by eye:
 
 * the state-specific attention mask over the augmented sequence x~_t = (x_t; s_t)
   (Sec. 3.1, Eq. 2; Sec. 3.2, query blocks 1-6 and Eq. 3),
-* masked softmax attention in float64 (a library matmul is one step),
+* masked softmax attention in float64 (a library matmul is one step), optionally after
+  the rotary position embedding of queries and keys, with each shadow row at the position
+  it copies (Sec. 3.1),
 * prediction / confidence (Sec. 3.1, Eq. 1), the verification-outcome kernel
   (Sec. 3.2, Eq. 5), the guidance weight (Eq. 6), logit mixing (Eq. 7) and the
   three-state transition (Eq. 8), taken in the order of Algorithm 1.
@@ -19,7 +21,8 @@ and are therefore formed in float32 exactly as the kernel forms them:
 ``mix = ls + w * (lx - ls)`` with each operation rounded to float32 (the paper's
 ``w*lx + (1-w)*ls`` regrouped; see ``mix_logits``).
 
-Readings of points the paper leaves open (the readings below):
+Readings of points the paper leaves open (numbered as in the project's full list of
+readings, whose other entries concern the workloads and the decoding driver):
   R1  keys of M positions seen by C queries and by M shadow queries come from s;
   R2  a shadow query s^i always sees its own shadow key s^i (no self leak), an original
       query x^i always sees x^i;
@@ -32,18 +35,23 @@ Readings of points the paper leaves open (the readings below):
       (NaN, +inf, or all -inf logits): confidence 0, token -1, state M;
   R7  a state byte above 2 is treated as M;
   R8  the attention scale is 1/sqrt(head_dim) unless given;
-  R9  p_cur, reported beside c, is the probability the scored distribution (shadow logits
+  R16 p_cur, reported beside c, is the probability the scored distribution (shadow logits
       for C and U positions, mixed logits for M positions) gives to the token currently at
       the position; 0 for a token outside the vocabulary or an invalid row;
-  R10 the token update that closes a step of Algorithm 1: positions that end the step in
+  R17 the token update that closes a step of Algorithm 1: positions that end the step in
       M hold the mask token again, every other position holds its new prediction x^;
-  R11 the ordering variants of the attention-mask ablation of Sec. 5 (bidirectional, l2r,
+  R18 the ordering variants of the attention-mask ablation of Sec. 5 (bidirectional, l2r,
       entropy, margin) differ only in the key that Eq. 3 compares: bidirectional = equal
       keys (every C pair attends both ways), l2r = minus the block position (earlier
       positions rank higher), entropy = minus the entropy of the scored distribution (in
       nats; more certain ranks higher), margin = p(x^) minus the second-largest probability
       (a repeated maximum gives 0; a one-entry vocabulary gives 1). An invalid row (R6) has
-      entropy 0 and margin 0.
+      entropy 0 and margin 0;
+  R20 the positional embedding is RoPE (the paper names none; its dLLMs use rotary
+      positions), applied to queries and keys before the masked attention; original row r
+      sits at position r and a shadow row at the position it copies (Sec. 3.1 only fixes
+      that the two copies share one positional embedding). Both common pairings of the
+      rotated elements are provided.
 
 Parity pins: every function here is pinned by ``tests/test_oracle_pins.py`` except where
 a docstring says "parity unpinned".
@@ -235,6 +243,49 @@ def masked_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, mask: np.ndarr
 
 
 # --------------------------------------------------------------------------------------
+# Rotary position embedding of the augmented sequence (Sec. 3.1)
+# --------------------------------------------------------------------------------------
+ROPE_INTERLEAVED, ROPE_HALF = 0, 1
+
+
+def row_positions(lay: SeqLayout) -> np.ndarray:
+    """Position of every row of x~_t (R20): the original copy x^r sits at r, and the shadow
+    copy s^j shares the positional embedding of x^j (Sec. 3.1), so shadow row N + k sits at
+    shadow_src[k]."""
+    return np.concatenate([np.arange(lay.n_orig, dtype=np.int64),
+                           np.asarray(lay.shadow_src, dtype=np.int64)])
+
+
+def rope(x: np.ndarray, positions: np.ndarray, theta: float,
+         style: int = ROPE_INTERLEAVED) -> np.ndarray:
+    """Rotary position embedding (Su et al., RoFormer, 2021) in float64 (R20).
+
+    x: [R, H, d]; positions: [R]. For frequency index i < d/2, f_i = theta^(-2i/d), and the
+    pair (a, b) of a row at position p becomes (a cos(p f_i) - b sin(p f_i),
+    a sin(p f_i) + b cos(p f_i)) in every head. The pairs are elements (2i, 2i+1)
+    (ROPE_INTERLEAVED) or (i, i + d/2) (ROPE_HALF). Returns float64 [R, H, d].
+    """
+    R, H, d = x.shape
+    i = np.arange(d // 2, dtype=np.float64)
+    freq = float(theta) ** (-2.0 * i / d)
+    ang = np.asarray(positions, dtype=np.float64)[:, None] * freq[None, :]  # [R, d/2]
+    cos = np.cos(ang)[:, None, :]
+    sin = np.sin(ang)[:, None, :]
+    x64 = x.astype(np.float64)
+    if style == ROPE_INTERLEAVED:
+        first, second = np.s_[..., 0::2], np.s_[..., 1::2]
+    elif style == ROPE_HALF:
+        first, second = np.s_[..., : d // 2], np.s_[..., d // 2:]
+    else:
+        raise ValueError(style)
+    a, b = x64[first], x64[second]
+    out = np.empty_like(x64)
+    out[first] = a * cos - b * sin
+    out[second] = a * sin + b * cos
+    return out
+
+
+# --------------------------------------------------------------------------------------
 # Scoring: confidence, mixing weight, logit mixing, state transition
 # --------------------------------------------------------------------------------------
 def confidence(logits_row: np.ndarray) -> tuple[float, int, bool]:
@@ -253,7 +304,7 @@ def confidence(logits_row: np.ndarray) -> tuple[float, int, bool]:
 
 
 def token_probability(logits_row: np.ndarray, tok: int) -> float:
-    """R9: softmax(logits)[tok] in float64, i.e. exp(l_tok - max) / sum exp(l - max).
+    """R16: softmax(logits)[tok] in float64, i.e. exp(l_tok - max) / sum exp(l - max).
 
     0.0 for tok outside [0, V) or an invalid row (R6).
     """
@@ -267,7 +318,7 @@ def token_probability(logits_row: np.ndarray, tok: int) -> float:
 
 
 def entropy(logits_row: np.ndarray) -> float:
-    """R11: -sum_v p_v ln p_v of the softmax of the row (float64); 0 for an invalid row."""
+    """R18: -sum_v p_v ln p_v of the softmax of the row (float64); 0 for an invalid row."""
     x = logits_row.astype(np.float64)
     if np.isnan(x).any() or np.isposinf(x).any() or np.isneginf(x).all():
         return 0.0
@@ -278,7 +329,7 @@ def entropy(logits_row: np.ndarray) -> float:
 
 
 def margin(logits_row: np.ndarray) -> float:
-    """R11: p(x^) minus the second-largest probability (float64); 0 for an invalid row."""
+    """R18: p(x^) minus the second-largest probability (float64); 0 for an invalid row."""
     x = logits_row.astype(np.float64)
     if np.isnan(x).any() or np.isposinf(x).any() or np.isneginf(x).all():
         return 0.0
@@ -290,18 +341,18 @@ def margin(logits_row: np.ndarray) -> float:
     return float(top[-1] - top[-2])
 
 
-# Ordering modes of R11 (the key Eq. 3 compares in the next step)
+# Ordering modes of R18 (the key Eq. 3 compares in the next step)
 ORDER_CONFIDENCE, ORDER_BIDIR, ORDER_L2R, ORDER_ENTROPY, ORDER_MARGIN = 0, 1, 2, 3, 4
 
 
 def order_key(mode: int, c: float, h: float, mg: float, i: int) -> float:
-    """R11: the next step's ordering key of block position i."""
+    """R18: the next step's ordering key of block position i."""
     return {ORDER_CONFIDENCE: c, ORDER_BIDIR: 0.0, ORDER_L2R: -float(i),
             ORDER_ENTROPY: -h, ORDER_MARGIN: mg}[mode]
 
 
 def next_tokens(token: np.ndarray, state_out: np.ndarray, mask_token: int) -> np.ndarray:
-    """R10, the last line of Algorithm 1's step: positions in C_{t+1} and U_{t+1} take the
+    """R17, the last line of Algorithm 1's step: positions in C_{t+1} and U_{t+1} take the
     decoded token x^, positions in M_{t+1} keep the mask token."""
     return np.where(np.asarray(state_out) == M, mask_token, np.asarray(token)).astype(np.int64)
 
@@ -352,10 +403,10 @@ class ScoreResult:
     promoted: list
     demoted: list
     counts: np.ndarray     # int64 [3]: M, C, U after the transition
-    p_cur: np.ndarray | None = None        # float64 [B] (R9), when cur_token is given
-    tokens_next: np.ndarray | None = None  # int64 [B] (R10), when mask_token is given
-    entropy: np.ndarray | None = None      # float64 [B] (R11) of each scored distribution
-    margin: np.ndarray | None = None       # float64 [B] (R11)
+    p_cur: np.ndarray | None = None        # float64 [B] (R16), when cur_token is given
+    tokens_next: np.ndarray | None = None  # int64 [B] (R17), when mask_token is given
+    entropy: np.ndarray | None = None      # float64 [B] (R18) of each scored distribution
+    margin: np.ndarray | None = None       # float64 [B] (R18)
 
 
 def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray,
@@ -369,8 +420,8 @@ def score_block(logits_x: np.ndarray, logits_s: np.ndarray, state_in: np.ndarray
     2. C positions move by Eq. 8; those that reach U form P, those that reach M form D.
     3. M positions: w from P and D (Eq. 5, 6), mixed logits (Eq. 7), c and x^ from them.
     4. M and U positions move by Eq. 8.
-    Optional: p_cur of cur_token on each scored distribution (R9), and the next step's
-    tokens (R10) when mask_token is given.
+    Optional: p_cur of cur_token on each scored distribution (R16), and the next step's
+    tokens (R17) when mask_token is given.
     """
     B = len(state_in)
     st = np.where(state_in > 2, M, state_in).astype(np.int64)  # R7

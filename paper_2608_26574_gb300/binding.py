@@ -33,7 +33,10 @@ class AttnArgs(ctypes.Structure):
                 ("block_len", _I32P), ("shadow_len", _I32P), ("state", ctypes.c_void_p),
                 ("prev_conf", ctypes.c_void_p), ("shadow_src", ctypes.c_void_p),
                 ("scale", ctypes.c_float), ("status", ctypes.c_void_p),
-                ("query_start", _I32P)]
+                ("query_start", _I32P), ("rope_theta", ctypes.c_float),
+                ("rope_style", ctypes.c_int32), ("k_rope", ctypes.c_void_p)]
+
+DARD_ROPE_INTERLEAVED, DARD_ROPE_HALF = 0, 1
 
 
 class ScoreArgs(ctypes.Structure):
@@ -184,10 +187,15 @@ class AttentionCall:
     calls it per layer. The host arrays are copied; the device tensors are referenced and
     must stay alive and unchanged in size while the object is used. Each call checks q, k,
     v and o against the row count the metadata implies (sum of n_orig + shadow_len), sets
-    the four pointers and the stream, and calls the library."""
+    the four pointers and the stream, and calls the library.
+
+    ``rope_theta`` > 0 makes the call apply RoPE (base theta, pairing ``rope_style``) to q
+    and k, which then arrive before RoPE; every call then needs ``k_rope``, a tensor shaped
+    like k that receives the rotated keys (k itself rotates k in place)."""
 
     def __init__(self, n_orig, block_start, block_len, shadow_len, state, prev_conf,
-                 shadow_src, scale: float = 0.0, status=None, query_start=None):
+                 shadow_src, scale: float = 0.0, status=None, query_start=None,
+                 rope_theta: float = 0.0, rope_style: int = DARD_ROPE_INTERLEAVED):
         torch = _torch()
         self._host = [_host_i32(x) for x in (n_orig, block_start, block_len, shadow_len)]
         self._qs = _host_i32(query_start) if query_start is not None else None
@@ -209,21 +217,25 @@ class AttentionCall:
         a.shadow_src = _dev(shadow_src, "shadow_src", sh, torch.int32, self.device)
         a.status = _dev(status, "status", 1, torch.int32, self.device)
         a.scale = scale
+        a.rope_theta = rope_theta
+        a.rope_style = rope_style
+        self.rope = rope_theta != 0.0
         self._keep = (state, prev_conf, shadow_src, status)
         self._args = a
         self._ref = ctypes.byref(a)
         self._fn = lib().dard_step_attention
 
-    def __call__(self, q, k, v, o, stream=None):
-        """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d]."""
-        dev = self._bind(q, k, v, o)
+    def __call__(self, q, k, v, o, stream=None, k_rope=None):
+        """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d]; with RoPE,
+        ``k_rope`` (like k) receives the rotated keys."""
+        dev = self._bind(q, k, v, o, k_rope)
         _check(self._fn(self._ref, _stream_handle(stream, dev)), "dard_step_attention")
 
     def kernel(self, q, k, v, o) -> int:
         """The kernel a call on these tensors launches, without launching it: 1 or 2 (the
         tensor-core kernel with one or two query tiles per CTA), 4 (the CTA-pair kernel),
         3 (fp32 CUDA cores), 0 (no query rows)."""
-        self._bind(q, k, v, o)
+        self._bind(q, k, v, o, k if self.rope else None)
         out = ctypes.c_int32(-1)
         _check(lib().dard_attention_kernel(self._ref, ctypes.byref(out)), "dard_attention_kernel")
         return int(out.value)
@@ -231,16 +243,16 @@ class AttentionCall:
     def plan(self, q, k, v, o) -> dict:
         """The launch plan of a call on these tensors, without launching it: the kernel, its
         CTAs, and the (query tile, key tile) pairs it computes and skips."""
-        self._bind(q, k, v, o)
+        self._bind(q, k, v, o, k if self.rope else None)
         out = AttnPlan()
         _check(lib().dard_attention_plan(self._ref, ctypes.byref(out)), "dard_attention_plan")
         return {"kernel": int(out.kernel), "ctas": int(out.ctas),
                 "tile_pairs": int(out.tile_pairs),
                 "tile_pairs_skipped": int(out.tile_pairs_skipped)}
 
-    def _bind(self, q, k, v, o) -> int:
-        """Checks q, k, v and o against the metadata and sets their pointers; returns the
-        device index."""
+    def _bind(self, q, k, v, o, k_rope=None) -> int:
+        """Checks q, k, v, o (and k_rope) against the metadata and sets their pointers;
+        returns the device index."""
         if not (q.is_cuda and k.is_cuda and v.is_cuda and o.is_cuda):
             raise ValueError("q, k, v and o must be device tensors")
         if not (q.is_contiguous() and k.is_contiguous() and v.is_contiguous()
@@ -259,8 +271,13 @@ class AttentionCall:
         if (k.get_device() != dev or v.get_device() != dev or o.get_device() != dev
                 or (self.device is not None and dev != self.device)):
             raise ValueError("q, k, v, o and the mask inputs need one device")
+        if k_rope is not None and (not k_rope.is_cuda or k_rope.shape != ks or
+                                   k_rope.dtype != dt or k_rope.get_device() != dev or
+                                   not k_rope.is_contiguous()):
+            raise ValueError("k_rope must be a contiguous device tensor like k")
         a = self._args
         a.q, a.k, a.v, a.o = q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr()
+        a.k_rope = k_rope.data_ptr() if k_rope is not None else None
         a.dtype = _dtype_code(q)
         a.hq, a.hkv, a.head_dim = qs[1], ks[1], qs[2]
         return dev
@@ -268,11 +285,14 @@ class AttentionCall:
 
 def dard_step_attention(q, k, v, o, n_orig, block_start, block_len, shadow_len, state,
                         prev_conf, shadow_src, scale: float = 0.0, status=None, stream=None,
-                        query_start=None):
+                        query_start=None, rope_theta: float = 0.0,
+                        rope_style: int = DARD_ROPE_INTERLEAVED, k_rope=None):
     """Masked attention of one layer; q/o [rows, hq, d], k/v [rows, hkv, d] on the device.
-    ``query_start`` (per sequence, optional): first query row; earlier rows are keys only."""
+    ``query_start`` (per sequence, optional): first query row; earlier rows are keys only.
+    ``rope_theta`` > 0: q and k arrive before RoPE, ``k_rope`` receives the rotated keys."""
     AttentionCall(n_orig, block_start, block_len, shadow_len, state, prev_conf, shadow_src,
-                  scale=scale, status=status, query_start=query_start)(q, k, v, o, stream)
+                  scale=scale, status=status, query_start=query_start, rope_theta=rope_theta,
+                  rope_style=rope_style)(q, k, v, o, stream, k_rope=k_rope)
 
 
 def dard_attention_kernel(q, k, v, o, n_orig, block_start, block_len, shadow_len, state,

@@ -52,7 +52,7 @@ const char* dard_status_string(dard_status s) {
 
 const char* dard_last_error(void) { return g_err; }
 
-int32_t dard_version(void) { return 20000; }
+int32_t dard_version(void) { return 20100; }
 
 }  // extern "C"
 
@@ -78,6 +78,15 @@ dard_status prepare_attention(const dard_attn_args* a, dard::AttnParams& p) {
     return fail(DARD_ERR_VALUE, "scale must be finite and >= 0");
   if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o))
     return fail(DARD_ERR_ALIGN, "q, k, v and o must be 16-byte aligned");
+  const bool rope = a->rope_theta != 0.f;
+  if (rope) {
+    if (!(a->rope_theta >= 1.f) || !std::isfinite(a->rope_theta))
+      return fail(DARD_ERR_VALUE, "rope_theta must be 0 or a finite value >= 1");
+    if (a->rope_style != DARD_ROPE_INTERLEAVED && a->rope_style != DARD_ROPE_HALF)
+      return fail(DARD_ERR_VALUE, "rope_style %d is not a dard_rope_style", a->rope_style);
+    if (!a->k_rope) return fail(DARD_ERR_NULL, "k_rope is NULL with rope_theta > 0");
+    if (!aligned16(a->k_rope)) return fail(DARD_ERR_ALIGN, "k_rope must be 16-byte aligned");
+  }
 
   memset(&p, 0, sizeof(p));
   long long rows = 0, blk = 0, sh = 0;
@@ -90,6 +99,9 @@ dard_status prepare_attention(const dard_attn_args* a, dard::AttnParams& p) {
     if (b0 < 0 || static_cast<long long>(b0) + B > n)
       return fail(DARD_ERR_SHAPE, "seq %d: block [%d, %d) outside [0, %d)", s, b0, b0 + B, n);
     if (S < 0 || S > B) return fail(DARD_ERR_SHAPE, "seq %d: shadow_len %d outside 0..%d", s, S, B);
+    if (rope && n > DARD_ROPE_MAX_POSITIONS)
+      return fail(DARD_ERR_SHAPE, "seq %d: n_orig %d exceeds the %d positions RoPE supports", s,
+                  n, DARD_ROPE_MAX_POSITIONS);
     const int qs = a->query_start ? a->query_start[s] : 0;
     if (qs < 0 || qs > n + S)
       return fail(DARD_ERR_SHAPE, "seq %d: query_start %d outside 0..%d", s, qs, n + S);
@@ -149,6 +161,20 @@ dard_status prepare_attention(const dard_attn_args* a, dard::AttnParams& p) {
   p.scale_log2 = p.scale * 1.4426950408889634f;
   p.wait_cycles = 0;
   p.test_drop_kv = -1;
+  p.k_src = a->k;
+  p.rope = rope ? 1 : 0;
+  if (rope) {
+    // f_i = theta^(-2i/D) in double, passed as a float and the float of its remainder
+    p.k = a->k_rope;
+    p.rope_style = a->rope_style;
+    for (int i = 0; i < a->head_dim / 2; ++i) {
+      const double f = std::pow(static_cast<double>(a->rope_theta),
+                                -2.0 * i / static_cast<double>(a->head_dim));
+      const float hi = static_cast<float>(f);
+      p.rope_f[2 * i] = hi;
+      p.rope_f[2 * i + 1] = static_cast<float>(f - static_cast<double>(hi));
+    }
+  }
   return DARD_OK;
 }
 

@@ -157,6 +157,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
     fence_barrier_init();
     tma_prefetch_desc(&tmk);
     tma_prefetch_desc(&tmv);
+    grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
     for (int j = 0; j < kNKV && j < n_kt; ++j) {
       load_kv(j, true);
       load_kv(j, false);
@@ -181,6 +182,19 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
 #pragma unroll
     for (int c = 0; c < D / 16; ++c)
       qhalf[c] = r < p.total_rows ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+    if (p.rope && q0 + t < rows_seq) {  // RoPE of this row (rows of the next sequence: unused)
+      const int pos = rope_position(p, sd, q0 + t);
+      if (p.rope_style == DARD_ROPE_INTERLEAVED) {
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c)
+          rope_chunk_interleaved(qhalf[c], pos, p.rope_f + 8 * (half * (D / 16) + c));
+      } else {  // the partner of each element is at the same offset of the other half
+        const uint4* other = src + (half == 0 ? D / 16 : -(D / 16));
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c)
+          rope_chunk_half(qhalf[c], __ldg(other + c), half == 0, pos, p.rope_f + 16 * c);
+      }
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -523,6 +537,7 @@ __device__ __forceinline__ void tile_row_exp(uint32_t tS, uint64_t vis0, uint64_
 // completion of use u - ring.
 struct __align__(16) Tc2Ctl {
   uint64_t q_full;  // both query tiles landed
+  uint64_t q_rot;   // RoPE: the softmax warps rotated the query tiles in shared memory
   uint64_t k_full[kNK], k_empty[kNK], v_full[kNV], v_empty[kNV];
   uint64_t s_full[kQT];   // S_q(j) landed in TMEM
   uint64_t p_full[kQT];   // the softmax of tile q stored P_q(j) over S_q(j)
@@ -545,7 +560,9 @@ __device__ __forceinline__ void flag_timeout(const AttnParams& p, Tc2Ctl& ctl) {
   if (p.status) atomicOr(p.status, DARD_STATUS_TIMEOUT);
 }
 
-template <int D>
+// kRope: the launch applies RoPE to the query tiles (a separate instantiation, so that the
+// kernel without RoPE keeps its register allocation).
+template <int D, bool kRope>
 __global__ void __launch_bounds__(kTc2Threads, 1)
     attn_tc2(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmq,
             const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv) {
@@ -593,6 +610,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   // K/V stages at once; the other threads touch the barriers only after the block sync.
   if (warp == kWProd && lane == 0) {
     mbar_init(&ctl.q_full, 1);
+    mbar_init(&ctl.q_rot, kQT * 4);  // the softmax warps
     for (int b = 0; b < kNK; ++b) {
       mbar_init(&ctl.k_full[b], 1);
       mbar_init(&ctl.k_empty[b], 1);
@@ -619,6 +637,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         tma_load_2d(sQ + q * kTileBytes + s * kKSub, &tmq, &ctl.q_full, h * D + s * 64,
                     row0 + sd.q_start + (qt0 + q) * kBM);
     }
+    grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
     for (int j = 0; j < kNK && j < n_kt; ++j) load_kv(j, true);
     for (int j = 0; j < kNV && j < n_kt; ++j) load_kv(j, false);
     for (int j = kNK; j < kNK + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
@@ -673,7 +692,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     if (lane == 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
       const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK);
-      bool ok = mbar_wait(&ctl.q_full, 0);
+      bool ok = mbar_wait(kRope ? &ctl.q_rot : &ctl.q_full, 0);
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
         ok = mbar_wait(&ctl.k_full[j % kNK], (j / kNK) & 1);
         for (int q = 0; q < nq && ok; ++q) {
@@ -730,6 +749,17 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     softmax_bar_sync();
     const int r = sd.q_start + (qt0 + q) * kBM + t;  // sequence-relative query row
     const bool active = q < nq;
+    if constexpr (kRope) {
+      // RoPE of this thread's query row in shared memory, before the first S product reads it
+      bool okq = mbar_wait(&ctl.q_full, 0);
+      okq = __all_sync(0xffffffffu, okq);
+      if (okq && active && r < rows_seq)
+        rope_tile_row<D>(p, sQ + q * kTileBytes, t, rope_position(p, sd, r));
+      if (!okq && lane == 0) flag_timeout(p, ctl);
+      fence_proxy_async_smem();  // the generic-proxy writes, before the MMAs read the tile
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.q_rot);
+    }
     const RowInfo ri = row_info(sd, ctl.bi, r);
     const RowMasks rm = row_masks(ri, ctl.bi, sd);
     const float sl = p.scale_log2;
@@ -873,6 +903,31 @@ __global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnPar
     qv[e] = live ? Q[qoff + 2 * e] : 0.f;
     acc[e] = 0.f;
   }
+  if (p.rope && live) {  // RoPE of this row; both threads of a row take this branch
+    const int pos = rope_position(p, sd, r);
+    if (p.rope_style == DARD_ROPE_INTERLEAVED) {
+      // pair e = elements (2e, 2e + 1): this thread holds one, its partner thread the other
+#pragma unroll
+      for (int e = 0; e < kH; ++e) {
+        float c, s;
+        rope_cos_sin(pos, p.rope_f[2 * e], p.rope_f[2 * e + 1], c, s);
+        const float other = __shfl_xor_sync(pair, qv[e], 1);
+        qv[e] = half == 0 ? fmaf(qv[e], c, -other * s) : fmaf(other, s, qv[e] * c);
+      }
+    } else {
+      // pair (i, i + D/2) with i = 2e + half: this thread's elements e and e + D/4
+#pragma unroll
+      for (int e = 0; e < kH / 2; ++e) {
+        const int i = 2 * e + half;
+        float c, s;
+        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
+        const float a = qv[e], b = qv[e + kH / 2];
+        qv[e] = fmaf(a, c, -b * s);
+        qv[e + kH / 2] = fmaf(a, s, b * c);
+      }
+    }
+  }
+  grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
   float m = -INFINITY, l = 0.f;
   for (int kt0 = 0; kt0 < rows_seq; kt0 += kKT) {
     __syncthreads();  // the previous tile has been read
@@ -959,7 +1014,7 @@ bool prefer_tc2(const AttnParams& p, int sms) {
 
 template <int D>
 cudaError_t launch_tc(const AttnParams& p, int kernel, cudaStream_t stream) {
-  static std::atomic<uint64_t> attr1_done{0}, attr2_done{0};
+  static std::atomic<uint64_t> attr1_done{0}, attr2_done{0}, attr2r_done{0};
   CUtensorMap mq, mk, mv;
   if (!make_map(&mk, p.k, p.hkv, D, p.total_rows, kTN) ||
       !make_map(&mv, p.v, p.hkv, D, p.total_rows, kTN))
@@ -967,16 +1022,19 @@ cudaError_t launch_tc(const AttnParams& p, int kernel, cudaStream_t stream) {
   if (kernel == 2) {
     if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM)) return cudaErrorInvalidValue;
     const size_t smem = tc2_smem_bytes<D>();
-    cudaError_t e = ensure_smem_attr(attn_tc2<D>, smem, attr2_done);
-    if (e != cudaSuccess) return e;
-    attn_tc2<D><<<p.total_pairs, kTc2Threads, smem, stream>>>(p, mq, mk, mv);
-  } else {
-    const size_t smem = tc1_smem_bytes<D>();
-    cudaError_t e = ensure_smem_attr(attn_tc1<D>, smem, attr1_done);
-    if (e != cudaSuccess) return e;
-    attn_tc1<D><<<p.total_work, kTc1Threads, smem, stream>>>(p, mk, mv);
+    const AttnLaunch L(p.total_pairs, kTc2Threads, smem, stream, 1, p.rope != 0);
+    if (p.rope) {
+      cudaError_t e = ensure_smem_attr(attn_tc2<D, true>, smem, attr2r_done);
+      return e != cudaSuccess ? e : cudaLaunchKernelEx(&L.cfg, attn_tc2<D, true>, p, mq, mk, mv);
+    }
+    cudaError_t e = ensure_smem_attr(attn_tc2<D, false>, smem, attr2_done);
+    return e != cudaSuccess ? e : cudaLaunchKernelEx(&L.cfg, attn_tc2<D, false>, p, mq, mk, mv);
   }
-  return cudaGetLastError();
+  const size_t smem = tc1_smem_bytes<D>();
+  cudaError_t e = ensure_smem_attr(attn_tc1<D>, smem, attr1_done);
+  if (e != cudaSuccess) return e;
+  const AttnLaunch L(p.total_work, kTc1Threads, smem, stream, 1, p.rope != 0);
+  return cudaLaunchKernelEx(&L.cfg, attn_tc1<D>, p, mk, mv);
 }
 
 }  // namespace
@@ -1005,10 +1063,17 @@ dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_
              cudaGetErrorString(cudaErrorLaunchFailure));
     return DARD_ERR_CUDA;
   }
+  if (p.rope) {  // the keys are rotated once, ahead of the attention kernel
+    e = launch_rope_keys(p, a.dtype, stream);
+    if (e != cudaSuccess) {
+      snprintf(err, err_len, "RoPE key pass launch failed: %s", cudaGetErrorString(e));
+      return DARD_ERR_CUDA;
+    }
+  }
   if (kernel == 3) {
-    if (a.head_dim == 64) attn_simt<64><<<p.total_work, 256, 0, stream>>>(p);
-    else attn_simt<128><<<p.total_work, 256, 0, stream>>>(p);
-    e = cudaGetLastError();
+    const AttnLaunch L(p.total_work, 256, 0, stream, 1, p.rope != 0);
+    e = a.head_dim == 64 ? cudaLaunchKernelEx(&L.cfg, attn_simt<64>, p)
+                         : cudaLaunchKernelEx(&L.cfg, attn_simt<128>, p);
   } else if (kernel == 4) {
     e = launch_pair_attention(p, stream);
   } else {

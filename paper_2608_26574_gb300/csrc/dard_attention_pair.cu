@@ -193,6 +193,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       int k_last[kPST], v_last[kPST];  // the latest use of each stage whose copy was issued
       for (int b = 0; b < kPST; ++b) k_last[b] = v_last[b] = -1;
       bool ok = true;
+      grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
       for (int w = cid; w < p.total_pairs && ok; w += ncl) {
         const PairItem it = pair_item(p, w);
         const int row0 = p.seq[it.seq].row_base;
@@ -343,20 +344,29 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         tma_load_2d(sO + kHalf, &tmq, &ctl.q_land, qi.h * D + 64, row);
       }
     };
-    // This thread's 32 elements of its query row (d = 32 slot .., four 16-byte chunks of row
-    // t in the staging buffer's swizzled block slot / 2) into TMEM (bf16 pairs), then tell
-    // rank 0.
-    auto store_q = [&]() -> bool {
+    // This thread's 32 elements of its query row in item qi (d = 32 slot .., 16-byte chunks
+    // 4 slot .. 4 slot + 3 of row t in the staging buffer), with RoPE when asked for, into
+    // TMEM (bf16 pairs), then tell rank 0.
+    auto store_q = [&](const PairItem& qi) -> bool {
       bool okq = mbar_wait(&ctl.q_land, q_loads & 1, wlim);
       okq = __all_sync(0xffffffffu, okq);
       ++q_loads;
       if (!okq) return false;
-      const uint8_t* src = sO + (slot >> 1) * kHalf + t * 128;
+      const SeqDesc& qsd = p.seq[qi.seq];
+      const int qr = qi.r0 + kBM * static_cast<int>(rank) + t;  // sequence-relative row
+      const bool rot = p.rope && qr < qsd.n_orig + qsd.slen;
+      const int pos = rot ? rope_position(p, qsd, qr) : 0;
       uint32_t qw[16];
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
-        const int chunk = (slot & 1) * 4 + c;
-        const uint4 u = *reinterpret_cast<const uint4*>(src + ((chunk ^ (t & 7)) << 4));
+        const int cg = 4 * slot + c;  // chunk of the row: elements 8 cg .. 8 cg + 7
+        uint4 u = *sw128_chunk(sO, t, cg);
+        if (rot) {
+          if (p.rope_style == DARD_ROPE_INTERLEAVED)
+            rope_chunk_interleaved(u, pos, p.rope_f + 8 * cg);
+          else  // the partner chunk D/2 elements away, in the other 64-column block
+            rope_chunk_half(u, *sw128_chunk(sO, t, cg ^ 8), cg < 8, pos, p.rope_f + 16 * (cg & 7));
+        }
         qw[4 * c + 0] = u.x;
         qw[4 * c + 1] = u.y;
         qw[4 * c + 2] = u.z;
@@ -376,7 +386,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       it = pair_item(p, w);
       load_q(it);
       if (warp < 4) bf = fetch_block_info(p, p.seq[it.seq]);
-      run = store_q();
+      run = store_q(it);
     }
     run = bar_and(2, kSoftmaxThreads, run);  // and every thread has read the staging buffer
     if (run && w + ncl < p.total_pairs) load_q(pair_item(p, w + ncl));
@@ -497,7 +507,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       // The item's last S has been read: the next item's Q may replace this one in TMEM,
       // so that its first S products run during this item's last PV and epilogue.
       bool go_on = ok && has_next;
-      if (go_on) go_on = store_q();
+      if (go_on) go_on = store_q(pair_item(p, w + ncl));
       // ---------------------------------------------------------- epilogue
       bool wok = ok && mbar_wait(&ctl.o_full, item_it & 1, wlim);
       wok = __all_sync(0xffffffffu, wok);
@@ -611,19 +621,8 @@ cudaError_t launch_pair_attention(const AttnParams& p, cudaStream_t stream) {
   const size_t smem = pair_smem_bytes();
   cudaError_t e = ensure_smem_attr(attn_pair, smem, attr_done);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2 * pair_clusters_for(p));
-  cfg.blockDim = dim3(kPairThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, attn_pair, p, mq, mk, mv);
+  const AttnLaunch L(2 * pair_clusters_for(p), kPairThreads, smem, stream, 2, p.rope != 0);
+  return cudaLaunchKernelEx(&L.cfg, attn_pair, p, mq, mk, mv);
 }
 
 }  // namespace dard

@@ -14,6 +14,7 @@
 
 #include "dard_internal.h"
 #include "dard_ptx.cuh"
+#include "dard_rope.cuh"
 
 namespace dard {
 namespace {
@@ -362,6 +363,39 @@ cudaError_t ensure_smem_attr(F* kernel, size_t bytes, std::atomic<uint64_t>& don
   if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
   return e;
 }
+// Launch configuration of an attention kernel: an optional cluster of `cluster` CTAs along
+// x, and programmatic dependent launch (pdl: the kernel may start while the RoPE key pass
+// launched before it is still running; its producer waits for that pass before any key
+// load). Not copyable: cfg points at attr.
+struct AttnLaunch {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[2];
+  AttnLaunch(unsigned grid, unsigned block, size_t smem, cudaStream_t stream, int cluster,
+             bool pdl) {
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    int n = 0;
+    if (cluster > 1) {
+      attr[n].id = cudaLaunchAttributeClusterDimension;
+      attr[n].val.clusterDim.x = cluster;
+      attr[n].val.clusterDim.y = 1;
+      attr[n].val.clusterDim.z = 1;
+      ++n;
+    }
+    if (pdl) {
+      attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+      attr[n].val.programmaticStreamSerializationAllowed = 1;
+      ++n;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = n;
+  }
+  AttnLaunch(const AttnLaunch&) = delete;
+  AttnLaunch& operator=(const AttnLaunch&) = delete;
+};
+
 int sm_count() {
   static std::atomic<int> cache[64];
   int dev = 0;

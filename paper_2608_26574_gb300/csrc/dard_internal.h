@@ -50,6 +50,12 @@ struct AttnParams {
   long long wait_cycles;     // bound of every in-kernel wait in SM cycles (0: the default)
   int32_t test_drop_kv;      // test hook: the K/V stage use whose K copy is never issued
                              // (a wait then runs out); -1 in normal operation
+  // RoPE (rope != 0): k is the rotated copy the key pass writes (k_rope of the call), k_src
+  // the keys as given; the attention kernels rotate q as they load it.
+  const void* k_src;
+  int32_t rope;
+  int32_t rope_style;        // DARD_ROPE_INTERLEAVED or DARD_ROPE_HALF
+  float rope_f[2 * 64];      // f_i = theta^(-2i/D) for i < D/2 as (float, remainder) pairs
   int32_t hq, hkv, head_dim, num_seqs;
   int32_t total_rows;
   int32_t total_work;        // number of (sequence, q-tile, head) work items
@@ -74,6 +80,10 @@ int pair_clusters_for(const AttnParams& p);
 
 dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
                              char* err, size_t err_len);
+
+// The RoPE pass over the key rows (rope != 0): k_src rotated into k. The attention kernel
+// launched after it on the same stream waits for it (programmatic dependent launch).
+cudaError_t launch_rope_keys(const AttnParams& p, int dtype, cudaStream_t stream);
 
 // ------------------------------------------------------------------ scoring
 struct ScoreParams {

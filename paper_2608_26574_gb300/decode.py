@@ -74,25 +74,11 @@ class DLLM:
                 w1=w(d, cfg.mlp, fan_in=d), w3=w(d, cfg.mlp, fan_in=d),
                 w2=w(cfg.mlp, d, fan_in=cfg.mlp)))
         self.head = w(d, cfg.vocab, fan_in=d)
-        inv = 1.0 / (cfg.rope_base ** (torch.arange(0, hd, 2, dtype=torch.float64) / hd))
-        self.inv_freq = inv.to(self.device)
 
     @staticmethod
     def rmsnorm(x):
         xf = x.float()
         return (xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + 1e-6)).to(x.dtype)
-
-    def rope(self, x, pos):
-        """Rotary embedding by position: pairs (2i, 2i+1) rotated by pos * inv_freq[i]."""
-        ang = pos.to(torch.float64)[:, None] * self.inv_freq[None, :]
-        cos = torch.cos(ang).float()[:, None, :]
-        sin = torch.sin(ang).float()[:, None, :]
-        xf = x.float()
-        a, b = xf[..., 0::2], xf[..., 1::2]
-        out = torch.empty_like(xf)
-        out[..., 0::2] = a * cos - b * sin
-        out[..., 1::2] = a * sin + b * cos
-        return out.to(x.dtype)
 
     def forward(self, batch: "Batch", need_attn_out: bool = False):
         """Logits of the block rows: (logits_x [sum B_i, V], logits_s [sum B_i, V])."""
@@ -100,17 +86,22 @@ class DLLM:
         rows = batch.tokens.numel()
         h = self.emb[batch.tokens.long()]
         attn_outs = []
-        # one step's mask metadata serves every layer: marshalled once
+        # one step's mask metadata serves every layer: marshalled once. RoPE runs inside the
+        # call (pairs (2i, 2i+1), base rope_base): q and k go in before RoPE, each row at its
+        # position and each shadow row at the position it copies; k_rope receives the keys.
         attention = B.AttentionCall(batch.n_orig, batch.block_start, batch.block_len,
                                     batch.shadow_len, batch.state, batch.prev_conf,
-                                    batch.shadow_src, status=batch.status)
+                                    batch.shadow_src, status=batch.status,
+                                    rope_theta=cfg.rope_base,
+                                    rope_style=B.DARD_ROPE_INTERLEAVED)
         for L in self.layers:
             a = self.rmsnorm(h)
-            q = self.rope((a @ L["wq"]).view(rows, cfg.hq, cfg.head_dim), batch.pos).contiguous()
-            k = self.rope((a @ L["wk"]).view(rows, cfg.hkv, cfg.head_dim), batch.pos).contiguous()
+            q = (a @ L["wq"]).view(rows, cfg.hq, cfg.head_dim).contiguous()
+            k = (a @ L["wk"]).view(rows, cfg.hkv, cfg.head_dim).contiguous()
             v = (a @ L["wv"]).view(rows, cfg.hkv, cfg.head_dim).contiguous()
             o = torch.empty_like(q)
-            attention(q, k, v, o)
+            k_rope = torch.empty_like(k)
+            attention(q, k, v, o, k_rope=k_rope)
             if need_attn_out:
                 attn_outs.append((q, k, v, o))
             h = h + o.view(rows, cfg.hq * cfg.head_dim) @ L["wo"]
@@ -130,7 +121,8 @@ class Batch:
     """Device state of one decoding step over a batch of sequences (paper layout: one
     shadow row per block position, shadow_src[k] = b0 + k)."""
     tokens: torch.Tensor      # int32 [rows]: x_t then s_t (mask tokens) per sequence
-    pos: torch.Tensor         # int32 [rows]: positions (shadow rows: their source position)
+    pos: torch.Tensor         # int32 [rows]: positions (shadow rows: their source position),
+                              # the ones dard_step_attention derives for RoPE
     n_orig: np.ndarray
     block_start: np.ndarray
     block_len: np.ndarray

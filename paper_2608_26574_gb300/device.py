@@ -38,7 +38,8 @@ class DeviceStep:
         sh = wl.shadow_src_all()
         self.shadow_src = torch.from_numpy(sh if len(sh) else np.zeros(1, np.int32)).to(dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
-        self._attn_calls: dict[float, B.AttentionCall] = {}
+        self._attn_calls: dict[tuple, B.AttentionCall] = {}
+        self._k_rope: dict[int, torch.Tensor] = {}
         self._score_calls: dict[tuple[bool, bool], B.ScoreCall] = {}
         self.layers = []
         if attention:
@@ -69,20 +70,35 @@ class DeviceStep:
             self.w_out = torch.empty(r, dtype=torch.float32, device=dev)
             self.counts = torch.empty(3 * len(wl.seqs), dtype=torch.int32, device=dev)
 
-    def attention_call(self, scale: float = 0.0) -> B.AttentionCall:
-        """The prepared attention call of this step (metadata marshalled once per scale)."""
-        c = self._attn_calls.get(scale)
+    def attention_call(self, scale: float = 0.0, rope=None) -> B.AttentionCall:
+        """The prepared attention call of this step (metadata marshalled once per scale and
+        RoPE setting; ``rope`` = (theta, style) or None)."""
+        key = (scale, rope)
+        c = self._attn_calls.get(key)
         if c is None:
+            theta, style = rope if rope is not None else (0.0, B.DARD_ROPE_INTERLEAVED)
             c = B.AttentionCall(self.n_orig, self.block_start, self.block_len, self.shadow_len,
                                 self.state, self.prev_conf, self.shadow_src, scale=scale,
-                                status=self.status, query_start=self.query_start)
-            self._attn_calls[scale] = c
+                                status=self.status, query_start=self.query_start,
+                                rope_theta=theta, rope_style=style)
+            self._attn_calls[key] = c
         return c
 
-    def attention(self, layer: int = 0, scale: float = 0.0, stream=None, out=None):
+    def k_rope(self, layer: int = 0) -> torch.Tensor:
+        """The buffer that receives a layer's rotated keys when RoPE is applied."""
+        t = self._k_rope.get(layer)
+        if t is None:
+            t = torch.empty_like(self.layers[layer][1])
+            self._k_rope[layer] = t
+        return t
+
+    def attention(self, layer: int = 0, scale: float = 0.0, stream=None, out=None, rope=None):
+        """One layer's attention; ``rope`` = (theta, style) applies RoPE in the call (the
+        rotated keys land in ``k_rope(layer)``)."""
         q, k, v, o = self.layers[layer]
         o = o if out is None else out
-        self.attention_call(scale)(q, k, v, o, stream)
+        kr = self.k_rope(layer) if rope is not None else None
+        self.attention_call(scale, rope)(q, k, v, o, stream, k_rope=kr)
         return o
 
     def score_call(self, w_out=True, counts=True, state_in=None) -> B.ScoreCall:

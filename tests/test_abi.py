@@ -80,6 +80,15 @@ def _attn_args(**kw):
     ({"b0": np.array([40], np.int32)}, 2), ({"sl": np.array([33], np.int32)}, 2),
     ({"b0": np.array([-1], np.int32)}, 2),
     ({"qs": np.array([97], np.int32)}, 2), ({"qs": np.array([-1], np.int32)}, 2),
+    # RoPE in the call: theta 0 or >= 1, a known pairing, a 16-byte aligned k_rope, and at
+    # most 2^20 positions per sequence
+    ({"rope_theta": 0.5, "k_rope": 0x30000}, 3), ({"rope_theta": -1.0, "k_rope": 0x30000}, 3),
+    ({"rope_theta": float("nan"), "k_rope": 0x30000}, 3),
+    ({"rope_theta": float("inf"), "k_rope": 0x30000}, 3),
+    ({"rope_theta": 1e4, "rope_style": 2, "k_rope": 0x30000}, 3),
+    ({"rope_theta": 1e4}, 1), ({"rope_theta": 1e4, "k_rope": 0x30008}, 6),
+    ({"rope_theta": 1e4, "k_rope": 0x30000, "n": np.array([(1 << 20) + 1], np.int32),
+      "b0": np.array([0], np.int32)}, 2),
 ])
 def test_attention_validation(lib, change, code):
     a, keep = _attn_args(**change)

@@ -318,8 +318,9 @@ def test_mask_probe_skipped_shadow_tiles(d, tc):
     torch.cuda.synchronize()
     mx, mean, n = P.compare_attention(wl, 0, o)
     # a wrongly skipped tile drops up to 64 attended keys of ~700 and moves a row's mean of
-    # N(0, 1) values by ~1e-2; the bf16 output rounding stays within half an ulp of |O|
-    tol = max(_probe_tol(wl), 3 * 2.0 ** -9 * float(abs(o).max()))
+    # N(0, 1) values by ~1e-2; the bf16 output rounding (half an ulp: at most 2^-8 of |O|)
+    # stays below 1.5 times that bound
+    tol = max(_probe_tol(wl), 1.5 * 2.0 ** -8 * float(abs(o).max()))
     print("skip probe", d, plan, mx, mean, n, tol)
     assert mx <= tol
     assert int(ds.status.item()) == 0

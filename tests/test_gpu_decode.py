@@ -43,16 +43,9 @@ def _cpu_forward(model, rec_tokens, batch, state, prev_conf):
         return x / np.sqrt((x * x).mean(-1, keepdims=True) + 1e-6)
 
     def rope(x, pos):
-        inv = 1.0 / (cfg.rope_base ** (np.arange(0, cfg.head_dim, 2) / cfg.head_dim))
-        ang = pos[:, None] * inv[None, :]
-        c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
-        a, b = x[..., 0::2], x[..., 1::2]
-        out = np.empty_like(x)
-        out[..., 0::2] = a * c - b * s
-        out[..., 1::2] = a * s + b * c
-        return out
+        return orc.rope(x, pos, cfg.rope_base, orc.ROPE_INTERLEAVED)
 
-    pos = batch.pos.cpu().numpy().astype(np.float64)
+    pos = batch.pos.cpu().numpy().astype(np.int64)
     h = _np(model.emb)[rec_tokens]
     rows = len(rec_tokens)
     nB = int(batch.block_len[0])
@@ -68,6 +61,8 @@ def _cpu_forward(model, rec_tokens, batch, state, prev_conf):
             lay = orc.SeqLayout(N, int(batch.block_start[si]), state[si * nB:(si + 1) * nB],
                                 prev_conf[si * nB:(si + 1) * nB],
                                 batch.shadow_src.cpu().numpy()[si * nB:(si + 1) * nB])
+            # the positions the library derives (R20) are the batch's
+            assert np.array_equal(orc.row_positions(lay), pos[sl])
             o[sl] = orc.masked_attention(q[sl], k[sl], v[sl], orc.attention_mask(lay))
         h = h + o.reshape(rows, -1) @ _np(L["wo"])
         m = rms(h)

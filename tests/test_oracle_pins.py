@@ -73,7 +73,7 @@ def test_eq2_exactly_one_copy_per_position(shadow):
 
 def test_all_unmasked_reduces_to_full_bidirectional():
     """With every token U and no candidates, original queries see every original key:
-    plain bidirectional attention over x (the benchmark spec's reduction; Sec. 3.2, U blocks)."""
+    plain bidirectional attention over x (Sec. 3.2, U blocks: U keys are taken in x)."""
     lay = _layout([U] * 6, [0.95] * 6, prompt=4, future=0)
     mask = orc.attention_mask(lay)
     n = lay.n_orig
@@ -280,7 +280,7 @@ def test_masked_attention_matches_library_sdpa_with_dense_mask():
 
 def test_attention_rows_are_convex_combinations():
     """Softmax weights are positive and sum to one: every output coordinate lies within the
-    range of the attended values (the benchmark spec invariant)."""
+    range of the attended values."""
     rng = np.random.default_rng(8)
     lay = _rand_layout(rng)
     R, hq, d = lay.rows, 2, 8
@@ -294,6 +294,124 @@ def test_attention_rows_are_convex_combinations():
         lo = v[att].min(axis=0) - 1e-12
         hi = v[att].max(axis=0) + 1e-12
         assert ((o[r] >= lo) & (o[r] <= hi)).all()
+
+
+# ---------------------------------------------------------------------------------------
+# RoPE of the augmented sequence (R20; Sec. 3.1: x^i and s^i share one position)
+# ---------------------------------------------------------------------------------------
+@pytest.mark.parametrize("style", [orc.ROPE_INTERLEAVED, orc.ROPE_HALF])
+def test_rope_position_zero_is_identity(style):
+    rng = np.random.default_rng(30)
+    x = rng.standard_normal((5, 3, 16))
+    assert np.array_equal(orc.rope(x, np.zeros(5, np.int64), 10000.0, style), x)
+
+
+def test_rope_single_pair_closed_form():
+    """d = 2: one pair at frequency theta^0 = 1, so position p turns (1, 0) into
+    (cos p, sin p) and (0, 1) into (-sin p, cos p), a counter-clockwise rotation by p."""
+    x = np.array([[[1.0, 0.0]], [[0.0, 1.0]], [[3.0, -2.0]]])
+    for p in (1, 2, 7, 100, 4095):
+        got = orc.rope(x, np.full(3, p), 500000.0)
+        c, s = math.cos(p), math.sin(p)
+        np.testing.assert_allclose(got[0, 0], [c, s], atol=1e-15)
+        np.testing.assert_allclose(got[1, 0], [-s, c], atol=1e-15)
+        np.testing.assert_allclose(got[2, 0], [3 * c + 2 * s, 3 * s - 2 * c], atol=1e-13)
+
+
+@pytest.mark.parametrize("style", [orc.ROPE_INTERLEAVED, orc.ROPE_HALF])
+def test_rope_frequency_of_each_pair(style):
+    """d = 8, theta = 16: pair i turns at f_i = 16^(-2i/8) = 2^(-i) radians per position.
+    A unit vector on the first element of pair i comes back as (cos(p 2^-i), sin(p 2^-i))
+    on that pair's two elements (2i, 2i+1 interleaved; i, i+4 half) and zero elsewhere."""
+    d, p = 8, 5
+    for i in range(d // 2):
+        a, b = (2 * i, 2 * i + 1) if style == orc.ROPE_INTERLEAVED else (i, i + d // 2)
+        x = np.zeros((1, 1, d))
+        x[0, 0, a] = 1.0
+        want = np.zeros(d)
+        want[a], want[b] = math.cos(p * 2.0 ** -i), math.sin(p * 2.0 ** -i)
+        np.testing.assert_allclose(orc.rope(x, np.array([p]), 16.0, style)[0, 0], want,
+                                   atol=1e-15)
+
+
+@pytest.mark.parametrize("style", [orc.ROPE_INTERLEAVED, orc.ROPE_HALF])
+def test_rope_preserves_every_pair_norm(style):
+    rng = np.random.default_rng(31)
+    d = 32
+    x = rng.standard_normal((40, 2, d))
+    pos = rng.integers(0, 1 << 20, size=40)
+    y = orc.rope(x, pos, 10000.0, style)
+    if style == orc.ROPE_INTERLEAVED:
+        nx = x[..., 0::2] ** 2 + x[..., 1::2] ** 2
+        ny = y[..., 0::2] ** 2 + y[..., 1::2] ** 2
+    else:
+        nx = x[..., :d // 2] ** 2 + x[..., d // 2:] ** 2
+        ny = y[..., :d // 2] ** 2 + y[..., d // 2:] ** 2
+    np.testing.assert_allclose(ny, nx, rtol=1e-12)
+
+
+def test_rope_scores_depend_on_position_differences():
+    """The defining property of RoPE, from complex arithmetic: with pair i read as
+    z = x_2i + j x_2i+1, <rope(q, p1), rope(k, p2)> = Re sum_i z_q conj(z_k) e^(j (p1-p2) f_i)."""
+    rng = np.random.default_rng(32)
+    d, theta = 16, 10000.0
+    q = rng.standard_normal((6, 1, d))
+    k = rng.standard_normal((6, 1, d))
+    p1 = rng.integers(0, 5000, size=6)
+    p2 = rng.integers(0, 5000, size=6)
+    got = (orc.rope(q, p1, theta) * orc.rope(k, p2, theta)).sum(-1)[:, 0]
+    zq = q[:, 0, 0::2] + 1j * q[:, 0, 1::2]
+    zk = k[:, 0, 0::2] + 1j * k[:, 0, 1::2]
+    f = np.array([theta ** (-2.0 * i / d) for i in range(d // 2)])
+    want = np.real((zq * np.conj(zk) * np.exp(1j * (p1 - p2)[:, None] * f)).sum(-1))
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-11)
+
+
+def test_rope_half_pairing_is_a_permuted_interleaved_pairing():
+    """Pairing (i, i + d/2) equals pairing (2i, 2i + 1) on the columns reordered as
+    0, d/2, 1, d/2 + 1, ..."""
+    rng = np.random.default_rng(33)
+    d = 12
+    x = rng.standard_normal((7, 3, d))
+    pos = rng.integers(0, 3000, size=7)
+    perm = np.ravel(np.column_stack([np.arange(d // 2), np.arange(d // 2) + d // 2]))
+    inter = orc.rope(x[..., perm], pos, 500000.0, orc.ROPE_INTERLEAVED)
+    back = np.empty_like(inter)
+    back[..., perm] = inter
+    np.testing.assert_allclose(orc.rope(x, pos, 500000.0, orc.ROPE_HALF), back, atol=1e-14)
+
+
+def test_row_positions_put_shadow_rows_at_their_source():
+    lay = _rand_layout(np.random.default_rng(34), B=10, prompt=6, future=3, shadow="candidates")
+    pos = orc.row_positions(lay)
+    assert np.array_equal(pos[:lay.n_orig], np.arange(lay.n_orig))
+    assert np.array_equal(pos[lay.n_orig:], lay.shadow_src)
+
+
+@pytest.mark.parametrize("style", [orc.ROPE_INTERLEAVED, orc.ROPE_HALF])
+def test_rope_attention_with_shared_positions(style):
+    """Two consequences pinned end to end. (1) Shifting every position by one constant
+    leaves the RoPE attention unchanged. (2) Shadow rows that carry the keys and values of
+    their source rows, rotated at their source positions, give plain RoPE attention over x
+    (library SDPA on the rotated original rows), as with no RoPE."""
+    rng = np.random.default_rng(35)
+    lay = _rand_layout(rng, B=10, prompt=9, future=6)
+    R, n, hq, hkv, d = lay.rows, lay.n_orig, 4, 2, 16
+    q = rng.standard_normal((R, hq, d))
+    k = rng.standard_normal((R, hkv, d))
+    v = rng.standard_normal((R, hkv, d))
+    pos = orc.row_positions(lay)
+    mask = orc.attention_mask(lay)
+    a = orc.masked_attention(orc.rope(q, pos, 100.0, style), orc.rope(k, pos, 100.0, style), v, mask)
+    b = orc.masked_attention(orc.rope(q, pos + 777, 100.0, style),
+                             orc.rope(k, pos + 777, 100.0, style), v, mask)
+    np.testing.assert_allclose(a, b, atol=1e-12)
+    k[n:] = k[lay.shadow_src]
+    v[n:] = v[lay.shadow_src]
+    qr, kr = orc.rope(q, pos, 100.0, style), orc.rope(k, pos, 100.0, style)
+    got = orc.masked_attention(qr, kr, v, mask)
+    want = _sdpa_torch(qr, kr[:n], v[:n])
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
 
 
 # ---------------------------------------------------------------------------------------
@@ -460,7 +578,7 @@ def test_score_block_fixed_weight_special_cases():
         assert res.token[r] == tok and abs(res.conf[r] - c) < 1e-15
 
 
-# ---------------------------------------------------------------- R9, R10 (p_cur, tokens)
+# ---------------------------------------------------------------- R16, R17 (p_cur, tokens)
 def test_token_probability_closed_forms():
     """A uniform row gives 1/V to every token; a planted row gives p to the peak and
     (1 - p)/(V - 1) to the rest (float32 rounding of the log only)."""
@@ -523,7 +641,7 @@ def test_next_tokens_fill_and_mask():
     assert list(res.tokens_next) == [4, 8, -7]
 
 
-# ---------------------------------------------------------------- R11 (ordering variants)
+# ---------------------------------------------------------------- R18 (ordering variants)
 def test_entropy_and_margin_closed_forms():
     V = 40
     u = np.zeros(V, np.float32)
@@ -554,7 +672,7 @@ def test_entropy_and_margin_against_library():
 
 
 def test_order_keys_reproduce_the_ablation_orderings():
-    """Eq. 3 with the R11 keys: equal keys make every C pair mutual (bidirectional); minus
+    """Eq. 3 with the R18 keys: equal keys make every C pair mutual (bidirectional); minus
     the position gives left-to-right causal order among C positions."""
     B = 6
     st = np.full(B, C, np.uint8)
