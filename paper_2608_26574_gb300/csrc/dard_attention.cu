@@ -46,7 +46,7 @@ namespace dard {
 namespace {
 
 constexpr int kTc1Threads = 352;  // attn_tc1: 8 softmax warps, producer, PV issuer, S issuer
-constexpr int kTc2Threads = 352;  // attn_tc2: 2 x 4 softmax warps, TMA producer, S and PV issuers
+constexpr int kTc2Threads = 384;  // attn_tc2: 2 x 4 softmax warps, TMA producer, S and PV issuers, spare
 
 constexpr int kQT = 2;   // query tiles per CTA (the same sequence and head)
 constexpr int kNK = 2;   // TMA stages for K
@@ -54,6 +54,14 @@ constexpr int kNV = 2;   // TMA stages for V
 constexpr int kWProd = 2 * kQT * 2;  // warp 8: TMA producer
 constexpr int kWMma = kWProd + 1;    // warp 9: TMEM allocator and S issuer
 constexpr int kWPv = kWProd + 2;     // warp 10: PV issuer
+// attn_tc2 register split (setmaxnreg): the launch gives 384 threads 168 registers each; the
+// warpgroup of warps 8-11 (producer, issuers, spare) drops to 56 and the two softmax
+// warpgroups rise to 224, so that a thread holds its row's 128 scores at once:
+// 128 x 56 + 256 x 224 = 384 x 168.
+constexpr uint32_t kTc2LaunchRegs = 168, kTc2SideRegs = 56, kTc2SoftmaxRegs = 224;
+static_assert(128 * kTc2SideRegs + 256 * kTc2SoftmaxRegs == kTc2Threads * kTc2LaunchRegs,
+              "the register shares must add up to the launch's registers");
+static_assert(kTc2Threads * kTc2LaunchRegs <= 65536, "one CTA per SM");
 
 // Named barriers: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = the 8 softmax warps,
 // then per kernel: attn_tc1 3 + q = the two warps sharing TMEM lane quarter q; attn_tc2
@@ -468,60 +476,49 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
 }
 
 
-// One query row's pass over a 128-key S tile in TMEM (columns tS .. tS + 127 of its lane),
-// 64 columns at a time; kMasked applies the visibility bits (vis0: keys 0-63, vis1: 64-127).
+// One query row's 128-key S tile out of TMEM (columns tS .. tS + 127 of its lane) into
+// registers, with the visibility bits applied (kMasked; vis0: keys 0-63, vis1: 64-127, a
+// hidden key becomes -inf); returns the row maximum. One wait for the four loads.
 template <bool kMasked>
-__device__ __forceinline__ float tile_row_max(uint32_t tS, uint64_t vis0, uint64_t vis1) {
+__device__ __forceinline__ float tile_row_load(uint32_t tS, uint64_t vis0, uint64_t vis1,
+                                               uint32_t (&sv)[128]) {
+#pragma unroll
+  for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(sv + 32 * c));
+  tmem_wait_ld();
+  if (kMasked) {
+#pragma unroll
+    for (int k = 0; k < 128; ++k) {
+      const uint64_t vis = k < 64 ? vis0 : vis1;
+      sv[k] = ((vis >> (k & 63)) & 1ull) ? sv[k] : 0xff800000u;  // -inf
+    }
+  }
   float mx[8];
 #pragma unroll
-  for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
+  for (int e = 0; e < 8; ++e)
+    mx[e] = fmax3(__uint_as_float(sv[e]), __uint_as_float(sv[8 + e]), __uint_as_float(sv[16 + e]));
 #pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
-    uint32_t r0[32], r1[32];
-    tmem_ld32(tS + 64 * hh, r0);
-    tmem_ld32(tS + 64 * hh + 32, r1);
-    tmem_wait_ld();
-    const uint64_t vis = hh ? vis1 : vis0;
+  for (int k = 24; k < 128; k += 16) {
 #pragma unroll
-    for (int e = 0; e < 32; e += 2) {
-      float x0 = __uint_as_float(r0[e]), x1 = __uint_as_float(r0[e + 1]);
-      float y0 = __uint_as_float(r1[e]), y1 = __uint_as_float(r1[e + 1]);
-      if (kMasked) {
-        x0 = ((vis >> e) & 1ull) ? x0 : -INFINITY;
-        x1 = ((vis >> (e + 1)) & 1ull) ? x1 : -INFINITY;
-        y0 = ((vis >> (32 + e)) & 1ull) ? y0 : -INFINITY;
-        y1 = ((vis >> (33 + e)) & 1ull) ? y1 : -INFINITY;
-      }
-      mx[(e >> 1) & 7] = fmaxf(fmax3(mx[(e >> 1) & 7], x0, x1), fmaxf(y0, y1));
-    }
+    for (int e = 0; e < 8; ++e)
+      mx[e] = k + 8 + e < 128 ? fmax3(mx[e], __uint_as_float(sv[k + e]), __uint_as_float(sv[k + 8 + e]))
+                              : fmaxf(mx[e], __uint_as_float(sv[k + e]));
   }
   return fmaxf(fmax3(mx[0], mx[1], mx[2]), fmax3(fmax3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
 }
 
-// P = 2^(s * sl - mL) for the row's 128 keys as bf16 pairs: keys 64 hh .. 64 hh + 63 go to
-// columns tS + 32 hh .. tS + 32 hh + 31, over S values this thread has already read. The
-// fp32 values are summed into acc (four packed partial sums).
-template <bool kMasked>
-__device__ __forceinline__ void tile_row_exp(uint32_t tS, uint64_t vis0, uint64_t vis1,
+// P = 2^(s * sl - mL) for the row's 128 scores held in registers, stored as bf16 pairs over
+// columns tS .. tS + 63 (the first half of the S tile's columns); the fp32 values are summed
+// into acc (four packed partial sums).
+__device__ __forceinline__ void tile_row_exp(uint32_t tS, const uint32_t (&sv)[128],
                                              uint64_t sl2, uint64_t nmL2, uint64_t (&acc)[4]) {
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
-    uint32_t r0[32], r1[32];
-    tmem_ld32(tS + 64 * hh, r0);
-    tmem_ld32(tS + 64 * hh + 32, r1);
-    tmem_wait_ld();
-    const uint64_t vis = hh ? vis1 : vis0;
     uint32_t pk[32];
 #pragma unroll
     for (int e = 0; e < 32; ++e) {
-      float s0 = __uint_as_float(e < 16 ? r0[2 * e] : r1[2 * e - 32]);
-      float s1 = __uint_as_float(e < 16 ? r0[2 * e + 1] : r1[2 * e - 31]);
-      if (kMasked) {
-        s0 = ((vis >> (2 * e)) & 1ull) ? s0 : -INFINITY;
-        s1 = ((vis >> (2 * e + 1)) & 1ull) ? s1 : -INFINITY;
-      }
       float x0, x1;
-      f2_unpack(f2_fma(f2_pack(s0, s1), sl2, nmL2), x0, x1);
+      f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[64 * hh + 2 * e]),
+                               __uint_as_float(sv[64 * hh + 2 * e + 1])), sl2, nmL2), x0, x1);
       const float a = ex2_approx(x0);
       const float c = ex2_approx(x1);
       acc[e & 3] = f2_add(acc[e & 3], f2_pack(a, c));
@@ -536,8 +533,8 @@ __device__ __forceinline__ void tile_row_exp(uint32_t tS, uint64_t vis0, uint64_
 // each wait for use u is preceded, in the same thread or through a chain of waits, by the
 // completion of use u - ring.
 struct __align__(16) Tc2Ctl {
-  uint64_t q_full;  // both query tiles landed
-  uint64_t q_rot;   // RoPE: the softmax warps rotated the query tiles in shared memory
+  uint64_t q_full[kQT];  // query tile q landed
+  uint64_t q_rot[kQT];   // RoPE: the softmax warps of tile q rotated it in shared memory
   uint64_t k_full[kNK], k_empty[kNK], v_full[kNV], v_empty[kNV];
   uint64_t s_full[kQT];   // S_q(j) landed in TMEM
   uint64_t p_full[kQT];   // the softmax of tile q stored P_q(j) over S_q(j)
@@ -606,11 +603,20 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       tma_prefetch_l2_2d(&tmv, g * D + s * 64, row0 + j * kTN);
     }
   };
-  // The producer lane initialises the barriers and issues the query tiles and the first
-  // K/V stages at once; the other threads touch the barriers only after the block sync.
+  auto load_q = [&](int q) {
+    mbar_arrive_expect_tx(&ctl.q_full[q], kTileBytes);
+#pragma unroll
+    for (int s = 0; s < kSub; ++s)
+      tma_load_2d(sQ + q * kTileBytes + s * kKSub, &tmq, &ctl.q_full[q], h * D + s * 64,
+                  row0 + sd.q_start + (qt0 + q) * kBM);
+  };
+  // The producer lane initialises the barriers and issues Q0 and K0; the other threads touch
+  // the barriers only after the block sync.
   if (warp == kWProd && lane == 0) {
-    mbar_init(&ctl.q_full, 1);
-    mbar_init(&ctl.q_rot, kQT * 4);  // the softmax warps
+    for (int q = 0; q < kQT; ++q) {
+      mbar_init(&ctl.q_full[q], 1);
+      mbar_init(&ctl.q_rot[q], 4);  // the tile's softmax warps
+    }
     for (int b = 0; b < kNK; ++b) {
       mbar_init(&ctl.k_full[b], 1);
       mbar_init(&ctl.k_empty[b], 1);
@@ -630,17 +636,11 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     tma_prefetch_desc(&tmq);
     tma_prefetch_desc(&tmk);
     tma_prefetch_desc(&tmv);
-    mbar_arrive_expect_tx(&ctl.q_full, nq * kTileBytes);
-    for (int q = 0; q < nq; ++q) {
-#pragma unroll
-      for (int s = 0; s < kSub; ++s)
-        tma_load_2d(sQ + q * kTileBytes + s * kKSub, &tmq, &ctl.q_full, h * D + s * 64,
-                    row0 + sd.q_start + (qt0 + q) * kBM);
-    }
+    // Q0 and K0 only: the first S product needs nothing else, and with every CTA of the
+    // launch starting at once they land sooner alone (the rest follows in the producer)
+    load_q(0);
     grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
-    for (int j = 0; j < kNK && j < n_kt; ++j) load_kv(j, true);
-    for (int j = 0; j < kNV && j < n_kt; ++j) load_kv(j, false);
-    for (int j = kNK; j < kNK + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
+    load_kv(0, true);
   }
   if (warp == kWMma) {
     tmem_alloc<kTmemCols>(&ctl.tmem_base);
@@ -657,10 +657,27 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   const uint32_t tO0 = ctl.tmem_base + kQT * kTN;
   volatile int32_t* abort_flag = &ctl.abort;
 
+  // The register split: each branch below starts with its warpgroup's setmaxnreg (warps 8-11
+  // give registers up, the softmax warps 0-7 take them), so that it covers the branch's code.
   if (warp == kWProd) {
     // ------------------------------------------------------------ TMA producer
+    reg_dealloc<kTc2SideRegs>();
     if (lane == 0) {
-      int last_k = min(n_kt, kNK) - 1, last_v = min(n_kt, kNV) - 1;
+      // the other first loads once Q0 and K0 have landed
+      int last_k = 0, last_v = -1, q_loaded = 1;
+      if (!mbar_wait(&ctl.q_full[0], 0) || !mbar_wait(&ctl.k_full[0], 0)) {
+        flag_timeout(p, ctl);
+      } else {
+        if (nq > 1) {
+          load_q(1);
+          q_loaded = 2;
+        }
+        load_kv(0, false);
+        last_v = 0;
+        for (int j = 1; j < kNK && j < n_kt; ++j) { load_kv(j, true); last_k = j; }
+        for (int j = 1; j < kNV && j < n_kt; ++j) { load_kv(j, false); last_v = j; }
+        for (int j = kNK; j < kNK + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
+      }
       for (int j = min(kNK, kNV); j < n_kt && !*abort_flag; ++j) {
         if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
         if (j >= kNK) {
@@ -680,11 +697,12 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         // let the copies already in flight land before shared memory is released
         if (last_k >= 0) mbar_wait(&ctl.k_full[last_k % kNK], (last_k / kNK) & 1);
         if (last_v >= 0) mbar_wait(&ctl.v_full[last_v % kNV], (last_v / kNV) & 1);
-        mbar_wait(&ctl.q_full, 0);
+        for (int q = 0; q < q_loaded; ++q) mbar_wait(&ctl.q_full[q], 0);
       }
     }
   } else if (warp == kWMma) {
     // ------------------------------------------------------------ S issuer
+    reg_dealloc<kTc2SideRegs>();
     // S_q(j) = Q_q K(j)^T once K(j) has landed and, for j > 0, PV_q(j - 1) has completed
     // (S_q(j) overwrites the P_q(j - 1) that PV_q(j - 1) reads). The PV products come from
     // a second issuer thread: one thread issuing both kinds of product in turn leaves the
@@ -692,11 +710,12 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     if (lane == 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
       const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK);
-      bool ok = mbar_wait(kRope ? &ctl.q_rot : &ctl.q_full, 0);
+      bool ok = true;
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
         ok = mbar_wait(&ctl.k_full[j % kNK], (j / kNK) & 1);
         for (int q = 0; q < nq && ok; ++q) {
-          if (j > 0) ok = mbar_wait(&ctl.pv_done[q], (j - 1) & 1);
+          if (j == 0) ok = mbar_wait(kRope ? &ctl.q_rot[q] : &ctl.q_full[q], 0);
+          else ok = mbar_wait(&ctl.pv_done[q], (j - 1) & 1);
           if (!ok) break;
           tc_fence_after();
           const uint32_t qaddr = aq + q * kTileBytes, kaddr = ak + (j % kNK) * kTileBytes;
@@ -714,6 +733,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     }
   } else if (warp == kWPv) {
     // ------------------------------------------------------------ PV issuer
+    reg_dealloc<kTc2SideRegs>();
     // O_q += P_q(j) V(j) once the softmax of tile q has stored P_q(j) and V(j) has landed.
     if (lane == 0) {
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
@@ -738,9 +758,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       }
       if (!ok) flag_timeout(p, ctl);
     }
-  } else {
+  } else if (warp < kWProd) {
     // ------------------------------------------------------------ softmax + epilogue
     // Warps 4q .. 4q + 3 own query tile q; thread t = query row t of the tile (TMEM lane t).
+    reg_alloc<kTc2SoftmaxRegs>();
     const int q = warp >> 2, quarter = warp & 3;
     const int t = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
@@ -749,16 +770,16 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     softmax_bar_sync();
     const int r = sd.q_start + (qt0 + q) * kBM + t;  // sequence-relative query row
     const bool active = q < nq;
-    if constexpr (kRope) {
+    if (kRope && active) {
       // RoPE of this thread's query row in shared memory, before the first S product reads it
-      bool okq = mbar_wait(&ctl.q_full, 0);
+      bool okq = mbar_wait(&ctl.q_full[q], 0);
       okq = __all_sync(0xffffffffu, okq);
-      if (okq && active && r < rows_seq)
+      if (okq && r < rows_seq)
         rope_tile_row<D>(p, sQ + q * kTileBytes, t, rope_position(p, sd, r));
       if (!okq && lane == 0) flag_timeout(p, ctl);
       fence_proxy_async_smem();  // the generic-proxy writes, before the MMAs read the tile
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.q_rot);
+      if (lane == 0) mbar_arrive(&ctl.q_rot[q]);
     }
     const RowInfo ri = row_info(sd, ctl.bi, r);
     const RowMasks rm = row_masks(ri, ctl.bi, sd);
@@ -772,9 +793,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       ok = !*abort_flag && mbar_wait(&ctl.s_full[q], j & 1);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
-      // pass 1: the row maximum over the tile's 128 keys
-      const float mt = masked ? tile_row_max<true>(tS + lane_off, vis0, vis1)
-                              : tile_row_max<false>(tS + lane_off, vis0, vis1);
+      // the tile's 128 scores of this row in registers, and their maximum
+      uint32_t sv[128];
+      const float mt = masked ? tile_row_load<true>(tS + lane_off, vis0, vis1, sv)
+                              : tile_row_load<false>(tS + lane_off, vis0, vis1, sv);
       // Raise the reference maximum on the first finite value, or when the tile maximum
       // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
       float m_new = m_run;
@@ -795,11 +817,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           tmem_st32(tO + lane_off + 32 * c, o);
         }
       }
-      // pass 2: P over the first 64 columns of S_q(j), and the row sum
+      // P over the first 64 columns of S_q(j), and the row sum
       const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
       uint64_t acc[4] = {0, 0, 0, 0};  // bit pattern 0 = +0.0f
-      if (masked) tile_row_exp<true>(tS + lane_off, vis0, vis1, sl2, nmL2, acc);
-      else tile_row_exp<false>(tS + lane_off, vis0, vis1, sl2, nmL2, acc);
+      tile_row_exp(tS + lane_off, sv, sl2, nmL2, acc);
       float a0, a1, b0, b1;
       f2_unpack(f2_add(acc[0], acc[1]), a0, a1);
       f2_unpack(f2_add(acc[2], acc[3]), b0, b1);
@@ -856,6 +877,8 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         }
       }
     }
+  } else {
+    reg_dealloc<kTc2SideRegs>();  // warp 11: completes the side warpgroup
   }
   tc_fence_before();
   __syncthreads();
@@ -1012,6 +1035,21 @@ bool prefer_tc2(const AttnParams& p, int sms) {
 }
 
 
+// attn_tc2's register split assumes a launch allocation of kTc2LaunchRegs per thread; with
+// any other, setmaxnreg.inc would wait for registers that never come. A build that allocated
+// otherwise is refused before its first launch (checked once per instantiation).
+template <class F>
+cudaError_t check_tc2_regs(F* kernel, std::atomic<int>& state) {
+  const int known = state.load(std::memory_order_acquire);
+  if (known != 0) return known == 1 ? cudaSuccess : cudaErrorInvalidDeviceFunction;
+  cudaFuncAttributes fa;
+  const cudaError_t e = cudaFuncGetAttributes(&fa, kernel);
+  if (e != cudaSuccess) return e;
+  const bool ok = fa.numRegs == static_cast<int>(kTc2LaunchRegs);
+  state.store(ok ? 1 : 2, std::memory_order_release);
+  return ok ? cudaSuccess : cudaErrorInvalidDeviceFunction;
+}
+
 template <int D>
 cudaError_t launch_tc(const AttnParams& p, int kernel, cudaStream_t stream) {
   static std::atomic<uint64_t> attr1_done{0}, attr2_done{0}, attr2r_done{0};
@@ -1022,12 +1060,15 @@ cudaError_t launch_tc(const AttnParams& p, int kernel, cudaStream_t stream) {
   if (kernel == 2) {
     if (!make_map(&mq, p.q, p.hq, D, p.total_rows, kBM)) return cudaErrorInvalidValue;
     const size_t smem = tc2_smem_bytes<D>();
+    static std::atomic<int> regs2{0}, regs2r{0};
     const AttnLaunch L(p.total_pairs, kTc2Threads, smem, stream, 1, p.rope != 0);
     if (p.rope) {
-      cudaError_t e = ensure_smem_attr(attn_tc2<D, true>, smem, attr2r_done);
+      cudaError_t e = check_tc2_regs(attn_tc2<D, true>, regs2r);
+      if (e == cudaSuccess) e = ensure_smem_attr(attn_tc2<D, true>, smem, attr2r_done);
       return e != cudaSuccess ? e : cudaLaunchKernelEx(&L.cfg, attn_tc2<D, true>, p, mq, mk, mv);
     }
-    cudaError_t e = ensure_smem_attr(attn_tc2<D, false>, smem, attr2_done);
+    cudaError_t e = check_tc2_regs(attn_tc2<D, false>, regs2);
+    if (e == cudaSuccess) e = ensure_smem_attr(attn_tc2<D, false>, smem, attr2_done);
     return e != cudaSuccess ? e : cudaLaunchKernelEx(&L.cfg, attn_tc2<D, false>, p, mq, mk, mv);
   }
   const size_t smem = tc1_smem_bytes<D>();

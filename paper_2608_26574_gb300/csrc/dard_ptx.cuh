@@ -316,6 +316,18 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 }
 
 // ---------------------------------------------------------------- misc
+// Register reallocation between the warpgroups of a CTA (every warp of a warpgroup executes
+// the same one): dec returns registers to the CTA's pool, inc waits until the pool holds
+// enough and takes them. The shares must add up to the launch's threads x registers.
+template <uint32_t kRegs>
+__device__ __forceinline__ void reg_alloc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegs));
+}
+template <uint32_t kRegs>
+__device__ __forceinline__ void reg_dealloc() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegs));
+}
+
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
