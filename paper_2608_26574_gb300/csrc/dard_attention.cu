@@ -1000,13 +1000,14 @@ __global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnPar
 
 // Which tensor-core kernel: a cost model in SM cycles, fitted (least squares on the log of
 // the time) to CUDA-graph timings of both kernels on the full and prefix-cached variants
-// of four workload shapes on GB300, within 5 % of each. attn_tc1 costs about
-// 14700 + 1480 kt cycles per 128-row query tile (kt = tiles of 128 keys); attn_tc2 about
-// 13900 + 3770 kt per pair of tiles and 8800 + 3000 kt for a lone last tile. Work spreads
-// over the SMs one CTA each: a launch with no more CTAs than SMs takes its longest CTA, a
-// larger one about total / SMs plus half a CTA of tail. attn_tc2 wins when few waves and
-// per-CTA setup dominate (8B layer: one wave instead of 1.5), attn_tc1 on long sequences
-// and on small query counts (prefix caching).
+// of four workload shapes on GB300 (within 6 % of each of the 16 timings). attn_tc1 costs
+// about 14250 + 1500 kt cycles per 128-row query tile (kt = tiles of 128 keys); attn_tc2
+// about 11900 + 3460 kt per pair of tiles and 32300 + 600 kt for a lone last tile (its
+// chain is latency-bound, much like a pair's). Work spreads over the SMs one CTA each: a
+// launch with no more CTAs than SMs takes its longest CTA, a larger one about total / SMs
+// plus half a CTA of tail. attn_tc2 wins on every full workload (8B layer: one wave instead
+// of 1.5, and its per-tile cost now below two of attn_tc1's), attn_tc1 on small query counts
+// (the 8B prefix-cached step); where the model errs (the GQA pair) the two differ by 1.5 %.
 struct TcEstimate {
   double total = 0, longest = 0;
   long long ctas = 0;
@@ -1027,9 +1028,9 @@ bool prefer_tc2(const AttnParams& p, int sms) {
     const SeqDesc& sd = p.seq[s];
     const double kt = (sd.n_orig + sd.slen + kTN - 1) / kTN;
     const long long tiles = sd.n_qtiles, heads = p.hq;
-    one.add(tiles * heads, 14700.0 + 1480.0 * kt);
-    two.add((tiles / 2) * heads, 13900.0 + 3770.0 * kt);
-    two.add((tiles % 2) * heads, 8800.0 + 3000.0 * kt);
+    one.add(tiles * heads, 14250.0 + 1500.0 * kt);
+    two.add((tiles / 2) * heads, 11900.0 + 3460.0 * kt);
+    two.add((tiles % 2) * heads, 32300.0 + 600.0 * kt);
   }
   return two.cycles(sms) < one.cycles(sms);
 }
