@@ -54,45 +54,55 @@ __global__ void __launch_bounds__(kRopeThreads) rope_keys(const __grid_constant_
   const SeqDesc& sd = p.seq[seq_of_row(p, row)];
   const int pos = rope_position(p, sd, row - sd.row_base);
   const bool half = p.rope_style == DARD_ROPE_HALF;
+  // element offsets of the group within a head: [e0, e0 + 4) and [e1, e1 + 4)
+  const int e0 = half ? 4 * grp : 8 * grp;
+  const int e1 = half ? D / 2 + 4 * grp : 8 * grp + 4;
+  const T* src = static_cast<const T*>(p.k_src);
+  T* dst = static_cast<T*>(const_cast<void*>(p.k));
+  const int h0 = hb * kRopeHeads;
+  // every head's loads first (they are independent), then the rotations and the stores
+  float x[kRopeHeads][8];
+#pragma unroll
+  for (int hh = 0; hh < kRopeHeads; ++hh) {
+    if (h0 + hh >= p.hkv) break;
+    const size_t base = (static_cast<size_t>(row) * p.hkv + h0 + hh) * D;
+    if constexpr (sizeof(T) == 2) {
+      const uint2 u0 = *reinterpret_cast<const uint2*>(src + base + e0);
+      const uint2 u1 = *reinterpret_cast<const uint2*>(src + base + e1);
+      x[hh][0] = bf_lo(u0.x); x[hh][1] = bf_hi(u0.x); x[hh][2] = bf_lo(u0.y); x[hh][3] = bf_hi(u0.y);
+      x[hh][4] = bf_lo(u1.x); x[hh][5] = bf_hi(u1.x); x[hh][6] = bf_lo(u1.y); x[hh][7] = bf_hi(u1.y);
+    } else {
+      const float4 u0 = *reinterpret_cast<const float4*>(src + base + e0);
+      const float4 u1 = *reinterpret_cast<const float4*>(src + base + e1);
+      x[hh][0] = u0.x; x[hh][1] = u0.y; x[hh][2] = u0.z; x[hh][3] = u0.w;
+      x[hh][4] = u1.x; x[hh][5] = u1.y; x[hh][6] = u1.z; x[hh][7] = u1.w;
+    }
+  }
+  // the angles while the loads are in flight
   float c[4], s[4];
 #pragma unroll
   for (int e = 0; e < 4; ++e) {
     const int i = 4 * grp + e;  // frequency index
     rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c[e], s[e]);
   }
-  // element offsets of the group within a head: [e0, e0 + 4) and [e1, e1 + 4)
-  const int e0 = half ? 4 * grp : 8 * grp;
-  const int e1 = half ? D / 2 + 4 * grp : 8 * grp + 4;
-  const T* src = static_cast<const T*>(p.k_src);
-  T* dst = static_cast<T*>(const_cast<void*>(p.k));
-  const int h_end = min(p.hkv, (hb + 1) * kRopeHeads);
-  for (int h = hb * kRopeHeads; h < h_end; ++h) {
-    const size_t base = (static_cast<size_t>(row) * p.hkv + h) * D;
-    float x[8];
-    if constexpr (sizeof(T) == 2) {
-      const uint2 u0 = *reinterpret_cast<const uint2*>(src + base + e0);
-      const uint2 u1 = *reinterpret_cast<const uint2*>(src + base + e1);
-      x[0] = bf_lo(u0.x); x[1] = bf_hi(u0.x); x[2] = bf_lo(u0.y); x[3] = bf_hi(u0.y);
-      x[4] = bf_lo(u1.x); x[5] = bf_hi(u1.x); x[6] = bf_lo(u1.y); x[7] = bf_hi(u1.y);
-    } else {
-      const float4 u0 = *reinterpret_cast<const float4*>(src + base + e0);
-      const float4 u1 = *reinterpret_cast<const float4*>(src + base + e1);
-      x[0] = u0.x; x[1] = u0.y; x[2] = u0.z; x[3] = u0.w;
-      x[4] = u1.x; x[5] = u1.y; x[6] = u1.z; x[7] = u1.w;
-    }
+#pragma unroll
+  for (int hh = 0; hh < kRopeHeads; ++hh) {
+    if (h0 + hh >= p.hkv) break;
+    float* y = x[hh];
     if (half) {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) rot(x[e], x[4 + e], c[e], s[e]);
+      for (int e = 0; e < 4; ++e) rot(y[e], y[4 + e], c[e], s[e]);
     } else {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) rot(x[2 * e], x[2 * e + 1], c[e], s[e]);
+      for (int e = 0; e < 4; ++e) rot(y[2 * e], y[2 * e + 1], c[e], s[e]);
     }
+    const size_t base = (static_cast<size_t>(row) * p.hkv + h0 + hh) * D;
     if constexpr (sizeof(T) == 2) {
-      *reinterpret_cast<uint2*>(dst + base + e0) = make_uint2(bf_pack(x[0], x[1]), bf_pack(x[2], x[3]));
-      *reinterpret_cast<uint2*>(dst + base + e1) = make_uint2(bf_pack(x[4], x[5]), bf_pack(x[6], x[7]));
+      *reinterpret_cast<uint2*>(dst + base + e0) = make_uint2(bf_pack(y[0], y[1]), bf_pack(y[2], y[3]));
+      *reinterpret_cast<uint2*>(dst + base + e1) = make_uint2(bf_pack(y[4], y[5]), bf_pack(y[6], y[7]));
     } else {
-      *reinterpret_cast<float4*>(dst + base + e0) = make_float4(x[0], x[1], x[2], x[3]);
-      *reinterpret_cast<float4*>(dst + base + e1) = make_float4(x[4], x[5], x[6], x[7]);
+      *reinterpret_cast<float4*>(dst + base + e0) = make_float4(y[0], y[1], y[2], y[3]);
+      *reinterpret_cast<float4*>(dst + base + e1) = make_float4(y[4], y[5], y[6], y[7]);
     }
   }
 }
