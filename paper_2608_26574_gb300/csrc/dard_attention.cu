@@ -82,6 +82,7 @@ struct __align__(16) Tc1Ctl {
   uint64_t q_full, o_full, p_full, pv_done;
   uint64_t k_full[kNKV], k_empty[kNKV], v_full[kNKV], v_empty[kNKV];
   uint64_t s_full[kNS], s_free[kNS];
+  uint64_t drained;  // every product both issuers launched has completed (two commits)
   uint32_t tmem_base;
   int32_t abort;
   BlockInfo bi;
@@ -125,6 +126,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
   const int n_kt = key_tiles(sd, q0, min(q0 + kBM, rows_seq));  // shadow-only tiles skipped
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long wlim = p.wait_cycles > 0 ? p.wait_cycles : kWaitCycles;
 
   // The producer lane initialises the barriers and issues the first kNKV K/V tiles at
   // once; the other threads touch the barriers only after the block-wide sync below.
@@ -135,6 +137,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
     uint8_t* dst = (k_or_v ? sK : sV) + b * kKVBytes;
     const void* map = k_or_v ? static_cast<const void*>(&tmk) : static_cast<const void*>(&tmv);
     mbar_arrive_expect_tx(bar, kKVBytes);
+    if (k_or_v && j == p.test_drop_kv) return;  // test hook: this K copy is never issued
 #pragma unroll
     for (int s = 0; s < kSub; ++s)
       tma_load_2d(dst + s * kKSub, map, bar, g * D + s * 64, row0 + j * kTN);
@@ -148,6 +151,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
   };
   if (warp == kWProd && lane == 0) {
     mbar_init(&ctl.q_full, kSoftmaxWarps);  // each softmax warp writes half of its Q rows
+    mbar_init(&ctl.drained, 2);
     mbar_init(&ctl.o_full, 1);
     mbar_init(&ctl.p_full, kSoftmaxWarps);
     mbar_init(&ctl.pv_done, 1);
@@ -220,17 +224,25 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       for (int j = kNKV; j < n_kt && !*abort_flag; ++j) {
         const int b = j % kNKV, ph = ((j - kNKV) / kNKV) & 1;
         if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
-        if (!mbar_wait(&ctl.k_empty[b], ph)) { flag_timeout(p, ctl); break; }
+        if (!mbar_wait(&ctl.k_empty[b], ph, wlim)) { flag_timeout(p, ctl); break; }
         load_kv(j, true);
         last_k = j;
-        if (!mbar_wait(&ctl.v_empty[b], ph)) { flag_timeout(p, ctl); break; }
+        if (!mbar_wait(&ctl.v_empty[b], ph, wlim)) { flag_timeout(p, ctl); break; }
         load_kv(j, false);
         last_v = j;
       }
-      if (*abort_flag) {
-        // let the copies already in flight land before shared memory is released
-        if (last_k >= 0) mbar_wait(&ctl.k_full[last_k % kNKV], (last_k / kNKV) & 1);
-        if (last_v >= 0) mbar_wait(&ctl.v_full[last_v % kNKV], (last_v / kNKV) & 1);
+      {
+        // Every copy issued lands before shared memory is released (after a normal run they
+        // all have: the waits return at once): the latest use of each stage (earlier uses
+        // landed before their stage was reused). A copy the test hook dropped was never
+        // issued.
+        for (int b = 0; b < kNKV; ++b) {
+          const int jk = last_k - ((last_k - b) % kNKV + kNKV) % kNKV;
+          const int jv = last_v - ((last_v - b) % kNKV + kNKV) % kNKV;
+          if (last_k >= 0 && jk >= 0 && jk != p.test_drop_kv)
+            mbar_wait(&ctl.k_full[b], (jk / kNKV) & 1, wlim);
+          if (last_v >= 0 && jv >= 0) mbar_wait(&ctl.v_full[b], (jv / kNKV) & 1, wlim);
+        }
       }
     }
   } else if (warp == kWS) {
@@ -240,11 +252,11 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
     if (lane == 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kTN, 0, 0);
       const uint32_t ak = smem_u32(sK);
-      bool ok = mbar_wait(&ctl.q_full, 0);
+      bool ok = mbar_wait(&ctl.q_full, 0, wlim);
       for (int t2 = 0; t2 < n_kt && ok && !*abort_flag; ++t2) {
         const int kb = t2 % kNKV, sb = t2 % kNS;
-        if (t2 >= kNS) ok = mbar_wait(&ctl.s_free[sb], ((t2 - kNS) / kNS) & 1);
-        ok = ok && mbar_wait(&ctl.k_full[kb], (t2 / kNKV) & 1);
+        if (t2 >= kNS) ok = mbar_wait(&ctl.s_free[sb], ((t2 - kNS) / kNS) & 1, wlim);
+        ok = ok && mbar_wait(&ctl.k_full[kb], (t2 / kNKV) & 1, wlim);
         if (!ok) break;
         tc_fence_after();
         const uint32_t kaddr = ak + kb * kKVBytes;
@@ -258,6 +270,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
         mma_commit(&ctl.k_empty[kb]);
       }
       if (!ok) flag_timeout(p, ctl);
+      mma_commit(&ctl.drained);  // completes once every S product this thread issued has
     }
   } else if (warp == kWPV) {
     // ------------------------------------------------------------ PV issuer
@@ -268,7 +281,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       bool ok = true;
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
         const int vb = j % kNKV;
-        ok = mbar_wait(&ctl.p_full, j & 1) && mbar_wait(&ctl.v_full[vb], (j / kNKV) & 1);
+        ok = mbar_wait(&ctl.p_full, j & 1, wlim) && mbar_wait(&ctl.v_full[vb], (j / kNKV) & 1, wlim);
         if (!ok) break;
         tc_fence_after();
         const uint32_t vaddr = av + vb * kKVBytes;
@@ -281,6 +294,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
         if (j == n_kt - 1) mma_commit(&ctl.o_full);
       }
       if (!ok) flag_timeout(p, ctl);
+      mma_commit(&ctl.drained);  // completes once every PV product this thread issued has
     }
   } else {
     // ------------------------------------------------------------ softmax + epilogue
@@ -326,7 +340,10 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       const int kt0 = j * kTN + half * 64;  // this warp's 64 keys
       const bool masked = tile_needs_mask(sd, j * kTN);
       const uint64_t vis = masked ? vis64(sd, kt0, rm) : ~0ull;
-      ok = !*abort_flag && mbar_wait(&ctl.s_full[b], (j / kNS) & 1);
+      // Both warps of the rows wait for the same S_j with the same bound (no early leave on
+      // an abort flag), so they leave the loop together: a barrier completing between the two
+      // warps' deadlines (a product about a second late) is the only way they could part.
+      ok = mbar_wait(&ctl.s_full[b], (j / kNS) & 1, wlim);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       float s[64];
@@ -394,7 +411,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       }
       // P_j replaces P_{j-1}, and O may be rescaled, once PV_{j-1} has completed
       if (j > 0) {
-        ok = mbar_wait(&ctl.pv_done, (j - 1) & 1);
+        ok = mbar_wait(&ctl.pv_done, (j - 1) & 1, wlim);  // the same barrier for both warps
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
       }
@@ -418,7 +435,7 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl.p_full);
     }
-    if (ok) ok = mbar_wait(&ctl.o_full, 0);
+    if (ok) ok = mbar_wait(&ctl.o_full, 0, wlim);
     const bool wok = __all_sync(0xffffffffu, ok);
     if (!wok && lane == 0) flag_timeout(p, ctl);
     // O row / row sum -> bf16 into shared memory (the K stages are no longer read once
@@ -470,6 +487,9 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == kWPV) {
+    // no product is still writing TMEM (both issuers committed `drained` last)
+    if (lane == 0 && !mbar_wait(&ctl.drained, 0, wlim)) flag_timeout(p, ctl);
+    __syncwarp();
     tc_fence_after();
     tmem_dealloc<kTmemCols>(ctl.tmem_base);
   }
@@ -540,6 +560,7 @@ struct __align__(16) Tc2Ctl {
   uint64_t p_full[kQT];   // the softmax of tile q stored P_q(j) over S_q(j)
   uint64_t pv_done[kQT];  // PV_q(j) completed: S_q's columns may take S_q(j + 1)
   uint64_t o_full[kQT];   // the last PV_q completed
+  uint64_t drained;       // every product both issuers launched has completed (two commits)
   uint32_t tmem_base;
   int32_t abort;
   BlockInfo bi;
@@ -585,6 +606,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   const int g = h / (p.hq / p.hkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row0 = sd.row_base;
+  const long long wlim = p.wait_cycles > 0 ? p.wait_cycles : kWaitCycles;
 
   auto load_kv = [&](int j, bool k_or_v) {
     const int b = j % (k_or_v ? kNK : kNV);
@@ -592,6 +614,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     uint8_t* dst = (k_or_v ? sK : sV) + b * kTileBytes;
     const void* map = k_or_v ? static_cast<const void*>(&tmk) : static_cast<const void*>(&tmv);
     mbar_arrive_expect_tx(bar, kTileBytes);
+    if (k_or_v && j == p.test_drop_kv) return;  // test hook: this K copy is never issued
 #pragma unroll
     for (int s = 0; s < kSub; ++s)
       tma_load_2d(dst + s * kKSub, map, bar, g * D + s * 64, row0 + j * kTN);
@@ -617,6 +640,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       mbar_init(&ctl.q_full[q], 1);
       mbar_init(&ctl.q_rot[q], 4);  // the tile's softmax warps
     }
+    mbar_init(&ctl.drained, 2);
     for (int b = 0; b < kNK; ++b) {
       mbar_init(&ctl.k_full[b], 1);
       mbar_init(&ctl.k_empty[b], 1);
@@ -665,7 +689,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     if (lane == 0) {
       // the other first loads once Q0 and K0 have landed
       int last_k = 0, last_v = -1, q_loaded = 1;
-      if (!mbar_wait(&ctl.q_full[0], 0) || !mbar_wait(&ctl.k_full[0], 0)) {
+      if (!mbar_wait(&ctl.q_full[0], 0, wlim) || !mbar_wait(&ctl.k_full[0], 0, wlim)) {
         flag_timeout(p, ctl);
       } else {
         if (nq > 1) {
@@ -682,22 +706,32 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
         if (j >= kNK) {
           const int b = j % kNK;
-          if (!mbar_wait(&ctl.k_empty[b], ((j - kNK) / kNK) & 1)) { flag_timeout(p, ctl); break; }
+          if (!mbar_wait(&ctl.k_empty[b], ((j - kNK) / kNK) & 1, wlim)) { flag_timeout(p, ctl); break; }
           load_kv(j, true);
           last_k = j;
         }
         if (j >= kNV) {
           const int b = j % kNV;
-          if (!mbar_wait(&ctl.v_empty[b], ((j - kNV) / kNV) & 1)) { flag_timeout(p, ctl); break; }
+          if (!mbar_wait(&ctl.v_empty[b], ((j - kNV) / kNV) & 1, wlim)) { flag_timeout(p, ctl); break; }
           load_kv(j, false);
           last_v = j;
         }
       }
-      if (*abort_flag) {
-        // let the copies already in flight land before shared memory is released
-        if (last_k >= 0) mbar_wait(&ctl.k_full[last_k % kNK], (last_k / kNK) & 1);
-        if (last_v >= 0) mbar_wait(&ctl.v_full[last_v % kNV], (last_v / kNV) & 1);
-        for (int q = 0; q < q_loaded; ++q) mbar_wait(&ctl.q_full[q], 0);
+      {
+        // Every copy issued lands before shared memory is released (after a normal run they
+        // all have: the waits return at once): the latest use of each stage (earlier uses
+        // landed before their stage was reused). A copy the test hook dropped was never
+        // issued.
+        for (int b = 0; b < kNK; ++b) {
+          const int jk = last_k - ((last_k - b) % kNK + kNK) % kNK;
+          if (last_k >= 0 && jk >= 0 && jk != p.test_drop_kv)
+            mbar_wait(&ctl.k_full[b], (jk / kNK) & 1, wlim);
+        }
+        for (int b = 0; b < kNV; ++b) {
+          const int jv = last_v - ((last_v - b) % kNV + kNV) % kNV;
+          if (last_v >= 0 && jv >= 0) mbar_wait(&ctl.v_full[b], (jv / kNV) & 1, wlim);
+        }
+        for (int q = 0; q < q_loaded; ++q) mbar_wait(&ctl.q_full[q], 0, wlim);
       }
     }
   } else if (warp == kWMma) {
@@ -712,10 +746,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       const uint32_t aq = smem_u32(sQ), ak = smem_u32(sK);
       bool ok = true;
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
-        ok = mbar_wait(&ctl.k_full[j % kNK], (j / kNK) & 1);
+        ok = mbar_wait(&ctl.k_full[j % kNK], (j / kNK) & 1, wlim);
         for (int q = 0; q < nq && ok; ++q) {
-          if (j == 0) ok = mbar_wait(kRope ? &ctl.q_rot[q] : &ctl.q_full[q], 0);
-          else ok = mbar_wait(&ctl.pv_done[q], (j - 1) & 1);
+          if (j == 0) ok = mbar_wait(kRope ? &ctl.q_rot[q] : &ctl.q_full[q], 0, wlim);
+          else ok = mbar_wait(&ctl.pv_done[q], (j - 1) & 1, wlim);
           if (!ok) break;
           tc_fence_after();
           const uint32_t qaddr = aq + q * kTileBytes, kaddr = ak + (j % kNK) * kTileBytes;
@@ -730,6 +764,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         if (ok) mma_commit(&ctl.k_empty[j % kNK]);
       }
       if (!ok) flag_timeout(p, ctl);
+      mma_commit(&ctl.drained);  // completes once every S product this thread issued has
     }
   } else if (warp == kWPv) {
     // ------------------------------------------------------------ PV issuer
@@ -740,9 +775,9 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       const uint32_t av = smem_u32(sV);
       bool ok = true;
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
-        ok = mbar_wait(&ctl.v_full[j % kNV], (j / kNV) & 1);
+        ok = mbar_wait(&ctl.v_full[j % kNV], (j / kNV) & 1, wlim);
         for (int q = 0; q < nq && ok; ++q) {
-          ok = mbar_wait(&ctl.p_full[q], j & 1);
+          ok = mbar_wait(&ctl.p_full[q], j & 1, wlim);
           if (!ok) break;
           tc_fence_after();
           const uint32_t vaddr = av + (j % kNV) * kTileBytes;
@@ -757,6 +792,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         if (ok) mma_commit(&ctl.v_empty[j % kNV]);
       }
       if (!ok) flag_timeout(p, ctl);
+      mma_commit(&ctl.drained);  // completes once every PV product this thread issued has
     }
   } else if (warp < kWProd) {
     // ------------------------------------------------------------ softmax + epilogue
@@ -772,7 +808,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     const bool active = q < nq;
     if (kRope && active) {
       // RoPE of this thread's query row in shared memory, before the first S product reads it
-      bool okq = mbar_wait(&ctl.q_full[q], 0);
+      bool okq = mbar_wait(&ctl.q_full[q], 0, wlim);
       okq = __all_sync(0xffffffffu, okq);
       if (okq && r < rows_seq)
         rope_tile_row<D>(p, sQ + q * kTileBytes, t, rope_position(p, sd, r));
@@ -790,7 +826,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       const bool masked = tile_needs_mask(sd, j * kTN);
       const uint64_t vis0 = masked ? vis64(sd, j * kTN, rm) : ~0ull;
       const uint64_t vis1 = masked ? vis64(sd, j * kTN + 64, rm) : ~0ull;
-      ok = !*abort_flag && mbar_wait(&ctl.s_full[q], j & 1);
+      ok = !*abort_flag && mbar_wait(&ctl.s_full[q], j & 1, wlim);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       // the tile's 128 scores of this row in registers, and their maximum
@@ -832,7 +868,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       if (lane == 0) mbar_arrive(&ctl.p_full[q]);
     }
     if (active) {
-      if (ok) ok = mbar_wait(&ctl.o_full[q], 0);
+      if (ok) ok = mbar_wait(&ctl.o_full[q], 0, wlim);
       const bool wok = __all_sync(0xffffffffu, ok);
       if (!wok && lane == 0) flag_timeout(p, ctl);
       // O row / row sum -> bf16 into the tile's query buffer (no MMA reads it once o_full
@@ -883,6 +919,9 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == kWMma) {
+    // no product is still writing TMEM (both issuers committed `drained` last)
+    if (lane == 0 && !mbar_wait(&ctl.drained, 0, wlim)) flag_timeout(p, ctl);
+    __syncwarp();
     tc_fence_after();
     tmem_dealloc<kTmemCols>(ctl.tmem_base);
   }

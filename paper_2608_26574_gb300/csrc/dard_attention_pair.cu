@@ -106,17 +106,6 @@ __device__ __forceinline__ PairItem pair_item(const AttnParams& p, int w) {
   return it;
 }
 
-// AND of `ok` over the threads of named barrier `id` (`n` threads), which it also syncs.
-__device__ __forceinline__ bool bar_and(int id, int n, bool ok) {
-  uint32_t r;
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
-      "barrier.red.and.pred q, %2, %3, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
-      : "=r"(r)
-      : "r"(static_cast<uint32_t>(ok)), "r"(id), "r"(n)
-      : "memory");
-  return r != 0;
-}
 
 // Named barrier 2 over every softmax thread of the CTA.
 __device__ __forceinline__ void softmax_sync() {

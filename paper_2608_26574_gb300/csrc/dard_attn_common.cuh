@@ -310,6 +310,18 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+// AND of `ok` over the threads of named barrier `id` (`n` threads), which it also syncs.
+__device__ __forceinline__ bool bar_and(int id, int n, bool ok) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+      "barrier.red.and.pred q, %2, %3, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(ok)), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
+}
+
 // Named barriers: 0 = __syncthreads, 1 = warps 0-3 (block info), 2 = the 8 softmax warps,
 // then per kernel 3 + q (see the kernel).
 __device__ __forceinline__ void softmax_bar_sync() {
@@ -319,6 +331,7 @@ __device__ __forceinline__ void softmax_bar_sync() {
 __device__ __forceinline__ void pair_bar_sync(int quarter) {
   asm volatile("bar.sync %0, 64;" ::"r"(3 + quarter) : "memory");
 }
+
 
 // ---------------------------------------------------------------- host side
 

@@ -48,7 +48,8 @@ struct AttnParams {
   float scale;               // softmax scale
   float scale_log2;          // scale * log2(e)
   long long wait_cycles;     // bound of every in-kernel wait in SM cycles (0: the default)
-  int32_t test_drop_kv;      // test hook: the K/V stage use whose K copy is never issued
+  int32_t test_drop_kv;      // test hook: the key tile (the CTA-pair kernel: the K stage use)
+                             // whose K copy is never issued
                              // (a wait then runs out); -1 in normal operation
   // RoPE (rope != 0): k is the rotated copy the key pass writes (k_rope of the call), k_src
   // the keys as given; the attention kernels rotate q as they load it.

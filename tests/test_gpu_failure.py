@@ -1,7 +1,7 @@
 """Failure paths, exercised without a GPU fault.
 
-An in-kernel wait that runs out: with a short wait bound (DARD_TEST_WAIT_CYCLES) the
-attention kernel on CTA pairs is told not to issue one K copy (DARD_TEST_DROP_KV; nothing
+An in-kernel wait that runs out: with a short wait bound (DARD_TEST_WAIT_CYCLES) each
+tensor-core attention kernel is told not to issue one K copy (DARD_TEST_DROP_KV; nothing
 invalid is issued, the copy simply never lands). Every wait that depends on it gives up,
 the launch ends with DARD_STATUS_TIMEOUT in the status word, and a normal call on the same
 device afterwards matches the oracle. An injected launch failure (DARD_TEST_FAIL_LAUNCH:
@@ -28,12 +28,15 @@ def _small(vocab=None):
     return W.custom(specs, 2, 2, 128, seed=5, **kw)
 
 
-def test_wait_runs_out_and_the_device_stays_usable(monkeypatch):
+@pytest.mark.parametrize("tc", ["1", "2", "4"])
+def test_wait_runs_out_and_the_device_stays_usable(monkeypatch, tc):
+    """Every tensor-core kernel: the one-tile and two-tile kernels drop the K copy of key
+    tile 1 in every CTA, the CTA-pair kernel the second K stage use of every pair."""
     wl = _small()
     ds = DeviceStep(wl, layers=[0], scoring=False)
-    monkeypatch.setenv("DARD_ATTN_TC", "4")
+    monkeypatch.setenv("DARD_ATTN_TC", tc)
     monkeypatch.setenv("DARD_TEST_WAIT_CYCLES", str(1 << 20))  # about half a millisecond
-    monkeypatch.setenv("DARD_TEST_DROP_KV", "1")  # the second K tile of every CTA pair
+    monkeypatch.setenv("DARD_TEST_DROP_KV", "1")
     ds.attention(0)
     torch.cuda.synchronize()
     assert int(ds.status.item()) & STATUS_TIMEOUT
