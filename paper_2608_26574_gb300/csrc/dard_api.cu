@@ -284,7 +284,7 @@ dard_status dard_attention_plan(const dard_attn_args* a, dard_attn_plan* plan) {
   if (p.total_work == 0) return DARD_OK;
   plan->kernel = attention_kernel_choice(*a, p);
   if (plan->kernel == 3) {
-    plan->ctas = p.total_work;
+    plan->ctas = static_cast<int64_t>(p.total_work) * kSimtCtasPerTile;
     return DARD_OK;
   }
   plan->ctas = plan->kernel == 1 ? p.total_work

@@ -928,28 +928,35 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
 }
 
 // ---------------------------------------------------------------- fp32 CUDA-core path
-// Two threads per query row (a CTA holds a 128-row query tile of one head): each owns the
-// row's even or odd elements of q and of the O accumulator in registers. The sequence's
-// keys pass through shared memory 32 rows at a time (K and V, read as broadcasts: the two
-// threads of a row read neighbouring words); per visible key the pair adds up its partial
-// dot products with one shuffle and updates its own online softmax. Masking as on the
-// tensor-core path, by key_visible().
+// A CTA holds 32 query rows of one head (a quarter of a 128-row query tile), four threads per
+// row, 128 threads: thread `part` of a row owns elements part, part + 4, ... of q and of the
+// O accumulator. The sequence's keys pass through shared memory 32 rows at a time (K and V,
+// read as broadcasts). Keys go four at a time: four independent partial dot products, which
+// the row's four threads add up with two shuffles each, then one online softmax step over
+// the four. Masking as on the tensor-core path, by key_visible().
+constexpr int kSimtRows = 32;     // query rows per CTA
+constexpr int kSimtParts = 4;     // threads per query row
+constexpr int kSimtThreads = kSimtRows * kSimtParts;
+constexpr int kSimtSplit = kSimtCtasPerTile;  // CTAs per 128-row query tile
+static_assert(kSimtSplit * kSimtRows == kBM, "the CTAs cover a 128-row query tile");
+
 template <int D>
-__global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnParams p) {
-  constexpr int kH = D / 2;  // elements per thread
-  constexpr int kKT = 32;    // keys per shared-memory tile
+__global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant__ AttnParams p) {
+  constexpr int kE = D / kSimtParts;  // elements per thread
+  constexpr int kKT = 32;             // keys per shared-memory tile
   __shared__ BlockInfo bi;
   __shared__ float sK[kKT][D], sV[kKT][D];
   int seq, qt, h;
-  decode_work(p, blockIdx.x, seq, qt, h);
+  decode_work(p, blockIdx.x / kSimtSplit, seq, qt, h);
+  const int sub = blockIdx.x % kSimtSplit;
   const SeqDesc sd = p.seq[seq];
   const int rows_seq = sd.n_orig + sd.slen;
   const int g = h / (p.hq / p.hkv);
-  if (threadIdx.x < 128) load_block_info(p, sd, bi, qt == 0 && h == 0);  // warps 0-3
+  load_block_info(p, sd, bi, qt == 0 && h == 0 && sub == 0);  // all 128 threads (warps 0-3)
   __syncthreads();
-  const int t = threadIdx.x >> 1, half = threadIdx.x & 1;
-  const unsigned pair = 3u << ((threadIdx.x & 31) & ~1);  // this thread and its partner
-  const int r = sd.q_start + qt * kBM + t;  // sequence-relative query row
+  const int t = threadIdx.x / kSimtParts, part = threadIdx.x % kSimtParts;
+  const unsigned quad = 0xfu << ((threadIdx.x & 31) & ~3);  // the row's four threads
+  const int r = sd.q_start + qt * kBM + sub * kSimtRows + t;  // sequence-relative query row
   const bool active = r < rows_seq;
   RowInfo q{0, kStateU, 0.f, -1, 0};
   if (active) q = row_info(sd, bi, r);
@@ -958,34 +965,35 @@ __global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnPar
   const float* K = static_cast<const float*>(p.k);
   const float* V = static_cast<const float*>(p.v);
   float* O = static_cast<float*>(p.o);
-  const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D + half;
-  float qv[kH], acc[kH];
+  const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D + part;
+  float qv[kE], acc[kE];
 #pragma unroll
-  for (int e = 0; e < kH; ++e) {
-    qv[e] = live ? Q[qoff + 2 * e] : 0.f;
+  for (int e = 0; e < kE; ++e) {
+    qv[e] = live ? Q[qoff + kSimtParts * e] : 0.f;
     acc[e] = 0.f;
   }
-  if (p.rope && live) {  // RoPE of this row; both threads of a row take this branch
+  if (p.rope && live) {  // RoPE of this row; the row's four threads take this branch together
     const int pos = rope_position(p, sd, r);
     if (p.rope_style == DARD_ROPE_INTERLEAVED) {
-      // pair e = elements (2e, 2e + 1): this thread holds one, its partner thread the other
+      // element 4e + part pairs with 4e + (part ^ 1), frequency 2e + part / 2
 #pragma unroll
-      for (int e = 0; e < kH; ++e) {
-        float c, s;
-        rope_cos_sin(pos, p.rope_f[2 * e], p.rope_f[2 * e + 1], c, s);
-        const float other = __shfl_xor_sync(pair, qv[e], 1);
-        qv[e] = half == 0 ? fmaf(qv[e], c, -other * s) : fmaf(other, s, qv[e] * c);
-      }
-    } else {
-      // pair (i, i + D/2) with i = 2e + half: this thread's elements e and e + D/4
-#pragma unroll
-      for (int e = 0; e < kH / 2; ++e) {
-        const int i = 2 * e + half;
+      for (int e = 0; e < kE; ++e) {
+        const int i = 2 * e + part / 2;
         float c, s;
         rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
-        const float a = qv[e], b = qv[e + kH / 2];
+        const float other = __shfl_xor_sync(quad, qv[e], 1);
+        qv[e] = (part & 1) == 0 ? fmaf(qv[e], c, -other * s) : fmaf(other, s, qv[e] * c);
+      }
+    } else {
+      // element d = 4e + part < D/2 pairs with d + D/2 = 4 (e + D/8) + part, frequency d
+#pragma unroll
+      for (int e = 0; e < kE / 2; ++e) {
+        const int i = kSimtParts * e + part;
+        float c, s;
+        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
+        const float a = qv[e], b = qv[e + kE / 2];
         qv[e] = fmaf(a, c, -b * s);
-        qv[e + kH / 2] = fmaf(a, s, b * c);
+        qv[e + kE / 2] = fmaf(a, s, b * c);
       }
     }
   }
@@ -993,7 +1001,7 @@ __global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnPar
   float m = -INFINITY, l = 0.f;
   for (int kt0 = 0; kt0 < rows_seq; kt0 += kKT) {
     __syncthreads();  // the previous tile has been read
-    for (int idx = threadIdx.x; idx < kKT * D; idx += 256) {
+    for (int idx = threadIdx.x; idx < kKT * D; idx += kSimtThreads) {
       const int kk = idx / D, d = idx % D;
       const int kr = kt0 + kk;
       float kx = 0.f, vx = 0.f;
@@ -1008,30 +1016,55 @@ __global__ void __launch_bounds__(256) attn_simt(const __grid_constant__ AttnPar
     __syncthreads();
     if (!live) continue;
     const int nk = min(kKT, rows_seq - kt0);
-    for (int kk = 0; kk < nk; ++kk) {
-      if (!key_visible(q, bi, sd, kt0 + kk)) continue;  // the same for both threads of a row
-      float dot = 0.f;
+    // four keys per step: four independent dot-product chains, one maximum and at most one
+    // rescale per step (keys past the sequence or hidden by the mask weigh 0)
+    for (int kk = 0; kk < nk; kk += 4) {
+      bool vis[4];
 #pragma unroll
-      for (int e = 0; e < kH; ++e) dot = fmaf(qv[e], sK[kk][2 * e + half], dot);
-      dot += __shfl_xor_sync(pair, dot, 1);
-      const float z = dot * p.scale;
-      if (z > m) {
-        const float alpha = (m == -INFINITY) ? 0.f : expf(m - z);
+      for (int u = 0; u < 4; ++u)
+        vis[u] = kk + u < nk && key_visible(q, bi, sd, kt0 + kk + u);  // the same for the row
+      if (!(vis[0] || vis[1] || vis[2] || vis[3])) continue;
+      float dot[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int e = 0; e < kE; ++e) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) dot[u] = fmaf(qv[e], sK[kk + u][kSimtParts * e + part], dot[u]);
+      }
+      float z[4];
+      float zmax = -INFINITY;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        dot[u] += __shfl_xor_sync(quad, dot[u], 1);
+        dot[u] += __shfl_xor_sync(quad, dot[u], 2);
+        z[u] = vis[u] ? dot[u] * p.scale : -INFINITY;
+        zmax = fmaxf(zmax, z[u]);
+      }
+      if (zmax > m) {
+        const float alpha = (m == -INFINITY) ? 0.f : expf(m - zmax);
         l *= alpha;
 #pragma unroll
-        for (int e = 0; e < kH; ++e) acc[e] *= alpha;
-        m = z;
+        for (int e = 0; e < kE; ++e) acc[e] *= alpha;
+        m = zmax;
       }
-      const float pz = expf(z - m);
-      l += pz;
+      float pz[4];
 #pragma unroll
-      for (int e = 0; e < kH; ++e) acc[e] = fmaf(pz, sV[kk][2 * e + half], acc[e]);
+      for (int u = 0; u < 4; ++u) {
+        pz[u] = vis[u] ? expf(z[u] - m) : 0.f;
+        l += pz[u];
+      }
+#pragma unroll
+      for (int e = 0; e < kE; ++e) {
+        float a = acc[e];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) a = fmaf(pz[u], sV[kk + u][kSimtParts * e + part], a);
+        acc[e] = a;
+      }
     }
   }
   if (live) {
     const float inv_l = 1.0f / l;
 #pragma unroll
-    for (int e = 0; e < kH; ++e) O[qoff + 2 * e] = acc[e] * inv_l;
+    for (int e = 0; e < kE; ++e) O[qoff + kSimtParts * e] = acc[e] * inv_l;
   }
 }
 
@@ -1152,7 +1185,7 @@ dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_
     }
   }
   if (kernel == 3) {
-    const AttnLaunch L(p.total_work, 256, 0, stream, 1, p.rope != 0);
+    const AttnLaunch L(p.total_work * kSimtSplit, kSimtThreads, 0, stream, 1, p.rope != 0);
     e = a.head_dim == 64 ? cudaLaunchKernelEx(&L.cfg, attn_simt<64>, p)
                          : cudaLaunchKernelEx(&L.cfg, attn_simt<128>, p);
   } else if (kernel == 4) {

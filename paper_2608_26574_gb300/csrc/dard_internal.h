@@ -26,6 +26,8 @@ struct SeqDesc {
 
 // Keys per tile of the tensor-core attention kernels.
 constexpr int kKeyTile = 128;
+// CTAs of the fp32 CUDA-core kernel per 128-row query tile (32 rows each).
+constexpr int kSimtCtasPerTile = 4;
 
 // Key tiles that query rows [r0, r1) of a sequence need. Original queries of positions after
 // the block (query block 1 of Sec. 3.2: M positions attend the x copy of every position) never
