@@ -107,6 +107,26 @@ __device__ __forceinline__ PairItem pair_item(const AttnParams& p, int w) {
 }
 
 
+// N (a multiple of 32) consecutive TMEM columns of this warp's lanes, from / to registers.
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t* r) {
+  static_assert(N % 32 == 0, "whole 32-column loads");
+#pragma unroll
+  for (int c = 0; c < N / 32; ++c)
+    tmem_ld32(taddr + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(r + 32 * c));
+}
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t* r) {
+  if constexpr (N == 16) {
+    tmem_st16(taddr, *reinterpret_cast<const uint32_t(*)[16]>(r));
+  } else {
+    static_assert(N % 32 == 0, "16 or whole 32-column stores");
+#pragma unroll
+    for (int c = 0; c < N / 32; ++c)
+      tmem_st32(taddr + 32 * c, *reinterpret_cast<const uint32_t(*)[32]>(r + 32 * c));
+  }
+}
+
 // Named barrier 2 over every softmax thread of the CTA.
 __device__ __forceinline__ void softmax_sync() {
   asm volatile("bar.sync 2, %0;" ::"n"(kSoftmaxThreads) : "memory");
@@ -333,9 +353,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         tma_load_2d(sO + kHalf, &tmq, &ctl.q_land, qi.h * D + 64, row);
       }
     };
-    // This thread's 32 elements of its query row in item qi (d = 32 slot .., 16-byte chunks
-    // 4 slot .. 4 slot + 3 of row t in the staging buffer), with RoPE when asked for, into
-    // TMEM (bf16 pairs), then tell rank 0.
+    // This thread's kCols elements of its query row in item qi (d = kCols slot .., 16-byte
+    // chunks of row t in the staging buffer), with RoPE when asked for, into TMEM (bf16
+    // pairs), then tell rank 0.
     auto store_q = [&](const PairItem& qi) -> bool {
       bool okq = mbar_wait(&ctl.q_land, q_loads & 1, wlim);
       okq = __all_sync(0xffffffffu, okq);
@@ -345,10 +365,10 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       const int qr = qi.r0 + kBM * static_cast<int>(rank) + t;  // sequence-relative row
       const bool rot = p.rope && qr < qsd.n_orig + qsd.slen;
       const int pos = rot ? rope_position(p, qsd, qr) : 0;
-      uint32_t qw[16];
+      uint32_t qw[kCols / 2];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int cg = 4 * slot + c;  // chunk of the row: elements 8 cg .. 8 cg + 7
+      for (int c = 0; c < kCols / 8; ++c) {
+        const int cg = (kCols / 8) * slot + c;  // chunk of the row: elements 8 cg .. 8 cg + 7
         uint4 u = *sw128_chunk(sO, t, cg);
         if (rot) {
           if (p.rope_style == DARD_ROPE_INTERLEAVED)
@@ -361,7 +381,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         qw[4 * c + 2] = u.z;
         qw[4 * c + 3] = u.w;
       }
-      tmem_st16(tQ + lane_off + slot * 16, qw);
+      tmem_st_cols<kCols / 2>(tQ + lane_off + slot * (kCols / 2), qw);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -402,56 +422,67 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       for (int j = 0; j < it.n_kt; ++j, ++tg) {
         const int b = tg & 1;
         const bool masked = tile_needs_mask(sd, j * kTN);
-        const uint32_t vis =
-            masked ? static_cast<uint32_t>(vis64(sd, j * kTN + kCols * slot, rm)) : ~0u;
+        // visibility of this thread's kCols keys (64 per word)
+        uint64_t vis[(kCols + 63) / 64];
+#pragma unroll
+        for (int c = 0; c < (kCols + 63) / 64; ++c)
+          vis[c] = masked ? vis64(sd, j * kTN + kCols * slot + 64 * c, rm) : ~0ull;
         bool wok = ok && !*abort_flag && mbar_wait(&ctl.s_full[b], (tg >> 1) & 1, wlim);
         wok = __all_sync(0xffffffffu, wok);
         float s[kCols];
         float mh = -INFINITY;
         if (wok) {
           tc_fence_after();
-          uint32_t r[32];
-          tmem_ld32(tS + b * kTN + kCols * slot + lane_off, r);
+          uint32_t r[kCols];
+          tmem_ld_cols<kCols>(tS + b * kTN + kCols * slot + lane_off, r);
           tmem_wait_ld();
           // S(t) is in registers: rank 0 may reuse its buffer for S(t + 2)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive_remote(lead(&ctl.s_free[b]));
 #pragma unroll
-          for (int e = 0; e < 32; ++e) s[e] = __uint_as_float(r[e]);
+          for (int e = 0; e < kCols; ++e) s[e] = __uint_as_float(r[e]);
           if (masked) {
 #pragma unroll
-            for (int k = 0; k < 32; ++k) s[k] = ((vis >> k) & 1u) ? s[k] : -INFINITY;
+            for (int k = 0; k < kCols; ++k)
+              s[k] = ((vis[k / 64] >> (k % 64)) & 1ull) ? s[k] : -INFINITY;
           }
           float mx[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) mx[e] = fmax3(s[e], s[8 + e], s[16 + e]);
+          for (int e = 0; e < 8; ++e) mx[e] = s[e];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[24 + e]);
+          for (int k = 8; k < kCols; k += 8) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[k + e]);
+          }
           mh = fmaxf(fmax3(mx[0], mx[1], mx[2]), fmax3(fmax3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
-          ctl.red_max[tg & 1][slot][t] = mh;
+          if (kSoftmaxSlots > 1) ctl.red_max[tg & 1][slot][t] = mh;
         }
-        // the four warps of the rows leave together, or all go on with all four maxima
+        // the warps of the rows leave together, or all go on with all their maxima
         if (!bar_and(3 + quarter, 32 * kSoftmaxSlots, wok)) {
           ok = false;
           break;
         }
-        const float mt = fmaxf(fmaxf(ctl.red_max[tg & 1][0][t], ctl.red_max[tg & 1][1][t]),
-                               fmaxf(ctl.red_max[tg & 1][2][t], ctl.red_max[tg & 1][3][t]));
+        float mt = mh;
+        if (kSoftmaxSlots > 1) {
+          mt = ctl.red_max[tg & 1][0][t];
+#pragma unroll
+          for (int sl2 = 1; sl2 < kSoftmaxSlots; ++sl2) mt = fmaxf(mt, ctl.red_max[tg & 1][sl2][t]);
+        }
         // Raise the reference maximum on the first finite value, or when the tile maximum
         // exceeds it by more than 2^kRescaleLog2 in probability; only then is O rescaled.
-        // The four warps of a row take the same decision from the same values.
+        // The warps of a row take the same decision from the same values.
         float m_new = m_run;
         if (m_run == -INFINITY) m_new = mt;
         else if ((mt - m_run) * sl > kRescaleLog2) m_new = mt;
         const bool rescale = (m_new != m_run) && (m_run != -INFINITY);
         const float alpha = rescale ? ex2_approx((m_run - m_new) * sl) : 1.f;
         const float mL = (m_new == -INFINITY) ? 0.f : m_new * sl;
-        uint32_t pk[16];
+        uint32_t pk[kCols / 2];
         const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
         uint64_t acc[2] = {0, 0};  // two packed partial sums (bit pattern 0 = +0.0f)
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
+        for (int e = 0; e < kCols / 2; ++e) {
           float x0, x1;
           f2_unpack(f2_fma(f2_pack(s[2 * e], s[2 * e + 1]), sl2, nmL2), x0, x1);
           pk[e] = pack_bf16x2(ex2_approx(x0), ex2_approx(x1));
@@ -471,12 +502,12 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           continue;
         }
         tc_fence_after();
-        tmem_st16(tP + lane_off + 16 * slot, pk);
+        tmem_st_cols<kCols / 2>(tP + lane_off + (kCols / 2) * slot, pk);
         // O (stable: PV(t - 1) completed, PV(t) waits for the arrival below) is rescaled
         // only when the reference maximum moved
         if (__any_sync(0xffffffffu, rescale)) {
 #pragma unroll 1
-          for (int c = 0; c < 2; ++c) {  // this warp's 32 O columns
+          for (int c = 0; c < kCols / 16; ++c) {  // this warp's kCols O columns
             uint32_t r[16];
             const uint32_t col = tO + lane_off + kCols * slot + 16 * c;
             tmem_ld16(col, r);
@@ -507,20 +538,25 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       uint4* stage = reinterpret_cast<uint4*>(sO);
       if (all_ok) {
         tc_fence_after();
-        const float inv_l =
-            1.0f / ((ctl.red_sum[0][t] + ctl.red_sum[1][t]) + (ctl.red_sum[2][t] + ctl.red_sum[3][t]));
-        uint32_t rr[32];
-        tmem_ld32(tO + lane_off + kCols * slot, rr);
-        tmem_wait_ld();
+        float lsum = ctl.red_sum[0][t];
 #pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          uint4 u;
-          u.x = pack_bf16x2(__uint_as_float(rr[8 * v + 0]) * inv_l, __uint_as_float(rr[8 * v + 1]) * inv_l);
-          u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
-          u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
-          u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
-          const int chunk = slot * 4 + v;
-          stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
+        for (int sl2 = 1; sl2 < kSoftmaxSlots; ++sl2) lsum += ctl.red_sum[sl2][t];
+        const float inv_l = 1.0f / lsum;
+#pragma unroll
+        for (int c = 0; c < kCols / 32; ++c) {  // this warp's kCols O columns, 32 at a time
+          uint32_t rr[32];
+          tmem_ld32(tO + lane_off + kCols * slot + 32 * c, rr);
+          tmem_wait_ld();
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 u;
+            u.x = pack_bf16x2(__uint_as_float(rr[8 * v + 0]) * inv_l, __uint_as_float(rr[8 * v + 1]) * inv_l);
+            u.y = pack_bf16x2(__uint_as_float(rr[8 * v + 2]) * inv_l, __uint_as_float(rr[8 * v + 3]) * inv_l);
+            u.z = pack_bf16x2(__uint_as_float(rr[8 * v + 4]) * inv_l, __uint_as_float(rr[8 * v + 5]) * inv_l);
+            u.w = pack_bf16x2(__uint_as_float(rr[8 * v + 6]) * inv_l, __uint_as_float(rr[8 * v + 7]) * inv_l);
+            const int chunk = slot * (kCols / 8) + 4 * c + v;
+            stage[t * kChunks + (chunk ^ (t & (kChunks - 1)))] = u;
+          }
         }
         // O has been read out: rank 0 may start the next item's first PV
         tc_fence_before();
