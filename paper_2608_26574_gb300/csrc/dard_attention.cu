@@ -14,7 +14,7 @@
 // attn_tc1: 128 query rows of one (sequence, head); 11 warps:
 //   warps 0-7  softmax and epilogue: warps w and w + 4 share TMEM lane quarter w (query
 //              rows 32w .. 32w + 31), each taking 64 of a tile's 128 key columns;
-//   warp 8     TMA producer: K and V through 3 stages each, L2 prefetches further ahead;
+//   warp 8     TMA producer: K and V through 3 stages each;
 //   warp 9     TMEM allocator and PV issuer: O += P_j V_j, P_j (bf16) read from TMEM;
 //   warp 10    S issuer: S_j = Q K_j^T (Q from TMEM, K from shared memory) into a ring of
 //              two 128-column TMEM buffers, reused once the softmax has read S_j.
@@ -142,13 +142,6 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
     for (int s = 0; s < kSub; ++s)
       tma_load_2d(dst + s * kKSub, map, bar, g * D + s * 64, row0 + j * kTN);
   };
-  auto prefetch_kv = [&](int j) {
-#pragma unroll
-    for (int s = 0; s < kSub; ++s) {
-      tma_prefetch_l2_2d(&tmk, g * D + s * 64, row0 + j * kTN);
-      tma_prefetch_l2_2d(&tmv, g * D + s * 64, row0 + j * kTN);
-    }
-  };
   if (warp == kWProd && lane == 0) {
     mbar_init(&ctl.q_full, kSoftmaxWarps);  // each softmax warp writes half of its Q rows
     mbar_init(&ctl.drained, 2);
@@ -174,7 +167,6 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       load_kv(j, true);
       load_kv(j, false);
     }
-    for (int j = kNKV; j < kNKV + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
   }
   if (warp == kWPV) {
     tmem_alloc<kTmemCols>(&ctl.tmem_base);
@@ -223,7 +215,6 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       int last_k = min(n_kt, kNKV) - 1, last_v = last_k;
       for (int j = kNKV; j < n_kt && !*abort_flag; ++j) {
         const int b = j % kNKV, ph = ((j - kNKV) / kNKV) & 1;
-        if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
         if (!mbar_wait(&ctl.k_empty[b], ph, wlim)) { flag_timeout(p, ctl); break; }
         load_kv(j, true);
         last_k = j;
@@ -619,13 +610,6 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     for (int s = 0; s < kSub; ++s)
       tma_load_2d(dst + s * kKSub, map, bar, g * D + s * 64, row0 + j * kTN);
   };
-  auto prefetch_kv = [&](int j) {
-#pragma unroll
-    for (int s = 0; s < kSub; ++s) {
-      tma_prefetch_l2_2d(&tmk, g * D + s * 64, row0 + j * kTN);
-      tma_prefetch_l2_2d(&tmv, g * D + s * 64, row0 + j * kTN);
-    }
-  };
   auto load_q = [&](int q) {
     mbar_arrive_expect_tx(&ctl.q_full[q], kTileBytes);
 #pragma unroll
@@ -700,10 +684,8 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         last_v = 0;
         for (int j = 1; j < kNK && j < n_kt; ++j) { load_kv(j, true); last_k = j; }
         for (int j = 1; j < kNV && j < n_kt; ++j) { load_kv(j, false); last_v = j; }
-        for (int j = kNK; j < kNK + kL2Ahead && j < n_kt; ++j) prefetch_kv(j);
       }
       for (int j = min(kNK, kNV); j < n_kt && !*abort_flag; ++j) {
-        if (j + kL2Ahead < n_kt) prefetch_kv(j + kL2Ahead);
         if (j >= kNK) {
           const int b = j % kNK;
           if (!mbar_wait(&ctl.k_empty[b], ((j - kNK) / kNK) & 1, wlim)) { flag_timeout(p, ctl); break; }
