@@ -484,9 +484,12 @@ __global__ void __launch_bounds__(kScoreThreads) score_pass2(const __grid_consta
   const int st = load_state(p, row, false);
   const int seq = seq_of_row(p, row);
   if (st != kStateM) {
-    if (split == 0 && p.counts != nullptr && threadIdx.x == 0) {
+    // The first row's first CTA waits for pass 1 even when nothing is counted, so that this
+    // grid cannot end before pass 1 has (also when no row is M): the call's last kernel
+    // ends after all of the call's work.
+    if (split == 0 && threadIdx.x == 0 && (p.counts != nullptr || row == 0)) {
       grid_dep_wait();
-      add_count(p, seq, __ldcg(p.state_out + row));
+      if (p.counts != nullptr) add_count(p, seq, __ldcg(p.state_out + row));
     }
     return;
   }
