@@ -382,24 +382,19 @@ __global__ void __launch_bounds__(kTc1Threads, 1)
       const float mL = (m_new == -INFINITY) ? 0.f : m_new * sl;
       uint32_t pk[32];
       const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
-      uint64_t acc[4] = {0, 0, 0, 0};  // four packed partial sums (bit pattern 0 = +0.0f)
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // partial sums
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
         float x0, x1;
         f2_unpack(f2_fma(f2_pack(s[2 * e], s[2 * e + 1]), sl2, nmL2), x0, x1);
-        const float a = ex2_approx(x0);
-        const float c = ex2_approx(x1);
-        const uint64_t pc = f2_pack(a, c);
-        acc[e & 3] = f2_add(acc[e & 3], pc);
-        pk[e] = pack_bf16x2(a, c);
+        pk[e] = pack_bf16x2(ex2_approx(x0), ex2_approx(x1));
+        // the row sum adds the rounded weights the PV product multiplies with (two
+        // mixed-precision adds: faster here than unpacking into a packed pair)
+        add_bf16x2_f32(acc[2 * (e & 3)], acc[2 * (e & 3) + 1], pk[e]);
       }
       float ls[4];
-      {
-        float a0, a1, b0, b1;
-        f2_unpack(f2_add(acc[0], acc[1]), a0, a1);
-        f2_unpack(f2_add(acc[2], acc[3]), b0, b1);
-        ls[0] = a0; ls[1] = a1; ls[2] = b0; ls[3] = b1;
-      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) ls[k] = acc[k] + acc[4 + k];
       // P_j replaces P_{j-1}, and O may be rescaled, once PV_{j-1} has completed
       if (j > 0) {
         ok = mbar_wait(&ctl.pv_done, (j - 1) & 1, wlim);  // the same barrier for both warps
@@ -518,8 +513,9 @@ __device__ __forceinline__ float tile_row_load(uint32_t tS, uint64_t vis0, uint6
 }
 
 // P = 2^(s * sl - mL) for the row's 128 scores held in registers, stored as bf16 pairs over
-// columns tS .. tS + 63 (the first half of the S tile's columns); the fp32 values are summed
-// into acc (four packed partial sums).
+// columns tS .. tS + 63 (the first half of the S tile's columns); the stored (rounded) values
+// are summed into acc (four packed partial sums), so that the output is a convex combination
+// of V rows with exactly the weights the PV product uses.
 __device__ __forceinline__ void tile_row_exp(uint32_t tS, const uint32_t (&sv)[128],
                                              uint64_t sl2, uint64_t nmL2, uint64_t (&acc)[4]) {
 #pragma unroll
@@ -530,10 +526,11 @@ __device__ __forceinline__ void tile_row_exp(uint32_t tS, const uint32_t (&sv)[1
       float x0, x1;
       f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[64 * hh + 2 * e]),
                                __uint_as_float(sv[64 * hh + 2 * e + 1])), sl2, nmL2), x0, x1);
-      const float a = ex2_approx(x0);
-      const float c = ex2_approx(x1);
-      acc[e & 3] = f2_add(acc[e & 3], f2_pack(a, c));
-      pk[e] = pack_bf16x2(a, c);
+      pk[e] = pack_bf16x2(ex2_approx(x0), ex2_approx(x1));
+      // the row sum adds the rounded weights the PV product multiplies with (unpacked by
+      // shift and mask into a packed pair: faster here than two mixed-precision adds)
+      acc[e & 3] = f2_add(acc[e & 3], f2_pack(__uint_as_float(pk[e] << 16),
+                                              __uint_as_float(pk[e] & 0xffff0000u)));
     }
     tmem_st32(tS + 32 * hh, pk);
   }
