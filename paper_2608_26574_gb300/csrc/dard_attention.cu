@@ -33,7 +33,7 @@
 //   O_0, O_1 [256, 256 + 2D).
 // Both keep a per-row running maximum and rescale O in TMEM only when the maximum grows by
 // more than a factor 2^8 (the exponentials stay bounded by 2^8 otherwise).
-// fp32 path (attn_simt): CUDA-core kernel, one warp per query row, same mask logic.
+// fp32 path: attn_simt (dard_attention_simt.cu), CUDA cores, the same mask logic.
 #include <algorithm>
 #include <cstdio>
 #include <cstdlib>
@@ -906,147 +906,6 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   }
 }
 
-// ---------------------------------------------------------------- fp32 CUDA-core path
-// A CTA holds 32 query rows of one head (a quarter of a 128-row query tile), four threads per
-// row, 128 threads: thread `part` of a row owns elements part, part + 4, ... of q and of the
-// O accumulator. The sequence's keys pass through shared memory 32 rows at a time (K and V,
-// read as broadcasts). Keys go four at a time: four independent partial dot products, which
-// the row's four threads add up with two shuffles each, then one online softmax step over
-// the four. Masking as on the tensor-core path, by key_visible().
-constexpr int kSimtRows = 32;     // query rows per CTA
-constexpr int kSimtParts = 4;     // threads per query row
-constexpr int kSimtThreads = kSimtRows * kSimtParts;
-constexpr int kSimtSplit = kSimtCtasPerTile;  // CTAs per 128-row query tile
-static_assert(kSimtSplit * kSimtRows == kBM, "the CTAs cover a 128-row query tile");
-
-template <int D>
-__global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant__ AttnParams p) {
-  constexpr int kE = D / kSimtParts;  // elements per thread
-  constexpr int kKT = 32;             // keys per shared-memory tile
-  __shared__ BlockInfo bi;
-  __shared__ float sK[kKT][D], sV[kKT][D];
-  int seq, qt, h;
-  decode_work(p, blockIdx.x / kSimtSplit, seq, qt, h);
-  const int sub = blockIdx.x % kSimtSplit;
-  const SeqDesc sd = p.seq[seq];
-  const int rows_seq = sd.n_orig + sd.slen;
-  const int g = h / (p.hq / p.hkv);
-  load_block_info(p, sd, bi, qt == 0 && h == 0 && sub == 0);  // all 128 threads (warps 0-3)
-  __syncthreads();
-  const int t = threadIdx.x / kSimtParts, part = threadIdx.x % kSimtParts;
-  const unsigned quad = 0xfu << ((threadIdx.x & 31) & ~3);  // the row's four threads
-  const int r = sd.q_start + qt * kBM + sub * kSimtRows + t;  // sequence-relative query row
-  const bool active = r < rows_seq;
-  RowInfo q{0, kStateU, 0.f, -1, 0};
-  if (active) q = row_info(sd, bi, r);
-  const bool live = active && q.store;
-  const float* Q = static_cast<const float*>(p.q);
-  const float* K = static_cast<const float*>(p.k);
-  const float* V = static_cast<const float*>(p.v);
-  float* O = static_cast<float*>(p.o);
-  const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D + part;
-  float qv[kE], acc[kE];
-#pragma unroll
-  for (int e = 0; e < kE; ++e) {
-    qv[e] = live ? Q[qoff + kSimtParts * e] : 0.f;
-    acc[e] = 0.f;
-  }
-  if (p.rope && live) {  // RoPE of this row; the row's four threads take this branch together
-    const int pos = rope_position(p, sd, r);
-    if (p.rope_style == DARD_ROPE_INTERLEAVED) {
-      // element 4e + part pairs with 4e + (part ^ 1), frequency 2e + part / 2
-#pragma unroll
-      for (int e = 0; e < kE; ++e) {
-        const int i = 2 * e + part / 2;
-        float c, s;
-        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
-        const float other = __shfl_xor_sync(quad, qv[e], 1);
-        qv[e] = (part & 1) == 0 ? fmaf(qv[e], c, -other * s) : fmaf(other, s, qv[e] * c);
-      }
-    } else {
-      // element d = 4e + part < D/2 pairs with d + D/2 = 4 (e + D/8) + part, frequency d
-#pragma unroll
-      for (int e = 0; e < kE / 2; ++e) {
-        const int i = kSimtParts * e + part;
-        float c, s;
-        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
-        const float a = qv[e], b = qv[e + kE / 2];
-        qv[e] = fmaf(a, c, -b * s);
-        qv[e + kE / 2] = fmaf(a, s, b * c);
-      }
-    }
-  }
-  grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
-  float m = -INFINITY, l = 0.f;
-  for (int kt0 = 0; kt0 < rows_seq; kt0 += kKT) {
-    __syncthreads();  // the previous tile has been read
-    for (int idx = threadIdx.x; idx < kKT * D; idx += kSimtThreads) {
-      const int kk = idx / D, d = idx % D;
-      const int kr = kt0 + kk;
-      float kx = 0.f, vx = 0.f;
-      if (kr < rows_seq) {
-        const size_t off = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D + d;
-        kx = K[off];
-        vx = V[off];
-      }
-      sK[kk][d] = kx;
-      sV[kk][d] = vx;
-    }
-    __syncthreads();
-    if (!live) continue;
-    const int nk = min(kKT, rows_seq - kt0);
-    // four keys per step: four independent dot-product chains, one maximum and at most one
-    // rescale per step (keys past the sequence or hidden by the mask weigh 0)
-    for (int kk = 0; kk < nk; kk += 4) {
-      bool vis[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        vis[u] = kk + u < nk && key_visible(q, bi, sd, kt0 + kk + u);  // the same for the row
-      if (!(vis[0] || vis[1] || vis[2] || vis[3])) continue;
-      float dot[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int e = 0; e < kE; ++e) {
-#pragma unroll
-        for (int u = 0; u < 4; ++u) dot[u] = fmaf(qv[e], sK[kk + u][kSimtParts * e + part], dot[u]);
-      }
-      float z[4];
-      float zmax = -INFINITY;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        dot[u] += __shfl_xor_sync(quad, dot[u], 1);
-        dot[u] += __shfl_xor_sync(quad, dot[u], 2);
-        z[u] = vis[u] ? dot[u] * p.scale : -INFINITY;
-        zmax = fmaxf(zmax, z[u]);
-      }
-      if (zmax > m) {
-        const float alpha = (m == -INFINITY) ? 0.f : expf(m - zmax);
-        l *= alpha;
-#pragma unroll
-        for (int e = 0; e < kE; ++e) acc[e] *= alpha;
-        m = zmax;
-      }
-      float pz[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        pz[u] = vis[u] ? expf(z[u] - m) : 0.f;
-        l += pz[u];
-      }
-#pragma unroll
-      for (int e = 0; e < kE; ++e) {
-        float a = acc[e];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) a = fmaf(pz[u], sV[kk + u][kSimtParts * e + part], a);
-        acc[e] = a;
-      }
-    }
-  }
-  if (live) {
-    const float inv_l = 1.0f / l;
-#pragma unroll
-    for (int e = 0; e < kE; ++e) O[qoff + kSimtParts * e] = acc[e] * inv_l;
-  }
-}
-
 // ---------------------------------------------------------------- host side
 
 // Which tensor-core kernel: a cost model in SM cycles, fitted (least squares on the log of
@@ -1164,9 +1023,7 @@ dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_
     }
   }
   if (kernel == 3) {
-    const AttnLaunch L(p.total_work * kSimtSplit, kSimtThreads, 0, stream, 1, p.rope != 0);
-    e = a.head_dim == 64 ? cudaLaunchKernelEx(&L.cfg, attn_simt<64>, p)
-                         : cudaLaunchKernelEx(&L.cfg, attn_simt<128>, p);
+    e = launch_simt_attention(p, stream);
   } else if (kernel == 4) {
     e = launch_pair_attention(p, stream);
   } else {

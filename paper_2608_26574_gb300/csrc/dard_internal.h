@@ -79,6 +79,9 @@ int attention_kernel_choice(const dard_attn_args& a, const AttnParams& p);
 // The pair kernel (two CTAs per 256-row work item, tcgen05 cta_group::2, head_dim 128,
 // persistent over work items): launch, and the number of clusters a launch uses.
 cudaError_t launch_pair_attention(const AttnParams& p, cudaStream_t stream);
+// The fp32 CUDA-core attention kernel (dard_attention_simt.cu); kSimtCtasPerTile CTAs per
+// 128-row query tile.
+cudaError_t launch_simt_attention(const AttnParams& p, cudaStream_t stream);
 int pair_clusters_for(const AttnParams& p);
 
 dard_status launch_attention(const dard_attn_args& a, AttnParams& p, cudaStream_t stream,
