@@ -88,22 +88,37 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
     }
   }
   grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
+  // K/V tiles are software-pipelined: each thread holds its share of the next tile in
+  // registers, loaded while the current tile is computed
+  constexpr int kLoads = kKT * D / kSimtThreads;  // elements of K (and of V) per thread
+  static_assert(kKT * D % kSimtThreads == 0, "a tile splits evenly over the threads");
+  float nxk[kLoads], nxv[kLoads];
+  auto fetch = [&](int kt0) {
+#pragma unroll
+    for (int u = 0; u < kLoads; ++u) {
+      const int idx = static_cast<int>(threadIdx.x) + u * kSimtThreads;
+      const int kr = kt0 + idx / D, d = idx % D;
+      nxk[u] = 0.f;
+      nxv[u] = 0.f;
+      if (kr < rows_seq) {
+        const size_t off = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D + d;
+        nxk[u] = K[off];
+        nxv[u] = V[off];
+      }
+    }
+  };
+  fetch(0);
   float m = -INFINITY, l = 0.f;
   for (int kt0 = 0; kt0 < rows_seq; kt0 += kKT) {
     __syncthreads();  // the previous tile has been read
-    for (int idx = threadIdx.x; idx < kKT * D; idx += kSimtThreads) {
-      const int kk = idx / D, d = idx % D;
-      const int kr = kt0 + kk;
-      float kx = 0.f, vx = 0.f;
-      if (kr < rows_seq) {
-        const size_t off = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D + d;
-        kx = K[off];
-        vx = V[off];
-      }
-      sK[kk][d] = kx;
-      sV[kk][d] = vx;
+#pragma unroll
+    for (int u = 0; u < kLoads; ++u) {
+      const int idx = static_cast<int>(threadIdx.x) + u * kSimtThreads;
+      sK[idx / D][idx % D] = nxk[u];
+      sV[idx / D][idx % D] = nxv[u];
     }
     __syncthreads();
+    if (kt0 + kKT < rows_seq) fetch(kt0 + kKT);
     if (!live) continue;
     const int k_end = min(kKT, rows_seq - kt0);
     // four keys per step: four independent dot-product chains, one maximum and at most one
