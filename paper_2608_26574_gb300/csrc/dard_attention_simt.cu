@@ -9,8 +9,10 @@ namespace {
 
 // ---------------------------------------------------------------- fp32 CUDA-core path
 // A CTA holds 32 query rows of one head (a quarter of a 128-row query tile), four threads per
-// row in each of four key groups, 512 threads: thread `part` of a row owns elements part,
-// part + 4, ... of q and of its O accumulator. The sequence's keys pass through shared
+// row in each of four key groups, 512 threads: thread `part` of a row owns the four-element
+// vectors 16 v + 4 part .. 16 v + 4 part + 3 (v = 0 .. D/16 - 1) of q and of its O
+// accumulator, so that the row's four threads read 64 contiguous bytes of a shared-memory
+// key row per vector (one 16-byte load each, no bank conflict). The sequence's keys pass through shared
 // memory 32 rows at a time (K and V, read as broadcasts); key group `grp` takes keys
 // 8 grp .. 8 grp + 7 of every tile, four at a time: four independent partial dot products,
 // which the row's four threads add up with two shuffles each, then one online softmax step
@@ -26,13 +28,14 @@ static_assert(kSimtSplit * kSimtRows == kBM, "the CTAs cover a 128-row query til
 
 template <int D>
 __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant__ AttnParams p) {
-  constexpr int kE = D / kSimtParts;           // elements per thread
+  constexpr int kV = D / 16;                   // float4 vectors per thread
   constexpr int kKT = 32;                      // keys per shared-memory tile
   constexpr int kKG = kKT / kSimtGroups;       // keys of a tile per key group
   static_assert(kKG % 4 == 0, "four keys per step");
   static_assert(kKT >= kSimtRows, "the merge reuses the K and V tile buffers, one row block each");
   __shared__ BlockInfo bi;
-  __shared__ float sK[kKT][D], sV[kKT][D];
+  __shared__ __align__(16) float sK[kKT][D];
+  __shared__ __align__(16) float sV[kKT][D];
   __shared__ float s_m[kSimtGroups][kSimtRows], s_l[kSimtGroups][kSimtRows];
   int seq, qt, h;
   decode_work(p, blockIdx.x / kSimtSplit, seq, qt, h);
@@ -55,55 +58,66 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
   const float* K = static_cast<const float*>(p.k);
   const float* V = static_cast<const float*>(p.v);
   float* O = static_cast<float*>(p.o);
-  const size_t qoff = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * D + part;
-  float qv[kE], acc[kE];
+  // vector v of this thread: float4 index 4 v + part of the row
+  const size_t qoff4 = (static_cast<size_t>(sd.row_base + r) * p.hq + h) * (D / 4) + part;
+  float4 qv[kV], acc[kV];
 #pragma unroll
-  for (int e = 0; e < kE; ++e) {
-    qv[e] = live ? Q[qoff + kSimtParts * e] : 0.f;
-    acc[e] = 0.f;
+  for (int v = 0; v < kV; ++v) {
+    qv[v] = live ? reinterpret_cast<const float4*>(Q)[qoff4 + 4 * v] : make_float4(0.f, 0.f, 0.f, 0.f);
+    acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  if (p.rope && live) {  // RoPE of this row; the row's four threads take this branch together
+  if (p.rope && live) {  // RoPE of this row; its pairs lie within one thread
     const int pos = rope_position(p, sd, r);
+    auto rot = [](float& a, float& b, float c, float s) {
+      const float x = a, y = b;
+      a = fmaf(x, c, -y * s);
+      b = fmaf(x, s, y * c);
+    };
     if (p.rope_style == DARD_ROPE_INTERLEAVED) {
-      // element 4e + part pairs with 4e + (part ^ 1), frequency 2e + part / 2
+      // elements (d, d + 1) of a vector, d = 16 v + 4 part + {0, 2}: frequency d / 2
 #pragma unroll
-      for (int e = 0; e < kE; ++e) {
-        const int i = 2 * e + part / 2;
-        float c, s;
-        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
-        const float other = __shfl_xor_sync(quad, qv[e], 1);
-        qv[e] = (part & 1) == 0 ? fmaf(qv[e], c, -other * s) : fmaf(other, s, qv[e] * c);
+      for (int v = 0; v < kV; ++v) {
+        const int i = 8 * v + 2 * part;
+        float c0, s0, c1, s1;
+        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c0, s0);
+        rope_cos_sin(pos, p.rope_f[2 * i + 2], p.rope_f[2 * i + 3], c1, s1);
+        rot(qv[v].x, qv[v].y, c0, s0);
+        rot(qv[v].z, qv[v].w, c1, s1);
       }
     } else {
-      // element d = 4e + part < D/2 pairs with d + D/2 = 4 (e + D/8) + part, frequency d
+      // element d = 16 v + 4 part + k < D/2 pairs with d + D/2 (vector v + kV/2): frequency d
 #pragma unroll
-      for (int e = 0; e < kE / 2; ++e) {
-        const int i = kSimtParts * e + part;
-        float c, s;
-        rope_cos_sin(pos, p.rope_f[2 * i], p.rope_f[2 * i + 1], c, s);
-        const float a = qv[e], b = qv[e + kE / 2];
-        qv[e] = fmaf(a, c, -b * s);
-        qv[e + kE / 2] = fmaf(a, s, b * c);
+      for (int v = 0; v < kV / 2; ++v) {
+        const int i = 16 * v + 4 * part;
+        float c[4], s[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) rope_cos_sin(pos, p.rope_f[2 * (i + k)], p.rope_f[2 * (i + k) + 1], c[k], s[k]);
+        float4& a = qv[v];
+        float4& b = qv[v + kV / 2];
+        rot(a.x, b.x, c[0], s[0]);
+        rot(a.y, b.y, c[1], s[1]);
+        rot(a.z, b.z, c[2], s[2]);
+        rot(a.w, b.w, c[3], s[3]);
       }
     }
   }
   grid_dep_wait();  // the RoPE key pass launched before this kernel (if any) is complete
   // K/V tiles are software-pipelined: each thread holds its share of the next tile in
   // registers, loaded while the current tile is computed
-  constexpr int kLoads = kKT * D / kSimtThreads;  // elements of K (and of V) per thread
-  static_assert(kKT * D % kSimtThreads == 0, "a tile splits evenly over the threads");
-  float nxk[kLoads], nxv[kLoads];
+  constexpr int kLoads = kKT * D / 4 / kSimtThreads;  // float4 of K (and of V) per thread
+  static_assert(kKT * D / 4 % kSimtThreads == 0, "a tile splits evenly over the threads");
+  float4 nxk[kLoads], nxv[kLoads];
   auto fetch = [&](int kt0) {
 #pragma unroll
     for (int u = 0; u < kLoads; ++u) {
       const int idx = static_cast<int>(threadIdx.x) + u * kSimtThreads;
-      const int kr = kt0 + idx / D, d = idx % D;
-      nxk[u] = 0.f;
-      nxv[u] = 0.f;
+      const int kr = kt0 + idx / (D / 4), c4 = idx % (D / 4);
+      nxk[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      nxv[u] = nxk[u];
       if (kr < rows_seq) {
-        const size_t off = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * D + d;
-        nxk[u] = K[off];
-        nxv[u] = V[off];
+        const size_t off = (static_cast<size_t>(sd.row_base + kr) * p.hkv + g) * (D / 4) + c4;
+        nxk[u] = reinterpret_cast<const float4*>(K)[off];
+        nxv[u] = reinterpret_cast<const float4*>(V)[off];
       }
     }
   };
@@ -114,8 +128,8 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
 #pragma unroll
     for (int u = 0; u < kLoads; ++u) {
       const int idx = static_cast<int>(threadIdx.x) + u * kSimtThreads;
-      sK[idx / D][idx % D] = nxk[u];
-      sV[idx / D][idx % D] = nxv[u];
+      reinterpret_cast<float4*>(sK[idx / (D / 4)])[idx % (D / 4)] = nxk[u];
+      reinterpret_cast<float4*>(sV[idx / (D / 4)])[idx % (D / 4)] = nxv[u];
     }
     __syncthreads();
     if (kt0 + kKT < rows_seq) fetch(kt0 + kKT);
@@ -131,9 +145,15 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
       if (!(vis[0] || vis[1] || vis[2] || vis[3])) continue;
       float dot[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int e = 0; e < kE; ++e) {
+      for (int v = 0; v < kV; ++v) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) dot[u] = fmaf(qv[e], sK[kk + u][kSimtParts * e + part], dot[u]);
+        for (int u = 0; u < 4; ++u) {
+          const float4 kx = reinterpret_cast<const float4*>(sK[kk + u])[4 * v + part];
+          dot[u] = fmaf(qv[v].x, kx.x, dot[u]);
+          dot[u] = fmaf(qv[v].y, kx.y, dot[u]);
+          dot[u] = fmaf(qv[v].z, kx.z, dot[u]);
+          dot[u] = fmaf(qv[v].w, kx.w, dot[u]);
+        }
       }
       float z[4];
       float zmax = -INFINITY;
@@ -148,7 +168,12 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
         const float alpha = (m == -INFINITY) ? 0.f : expf(m - zmax);
         l *= alpha;
 #pragma unroll
-        for (int e = 0; e < kE; ++e) acc[e] *= alpha;
+        for (int v = 0; v < kV; ++v) {
+          acc[v].x *= alpha;
+          acc[v].y *= alpha;
+          acc[v].z *= alpha;
+          acc[v].w *= alpha;
+        }
         m = zmax;
       }
       float pz[4];
@@ -158,11 +183,15 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
         l += pz[u];
       }
 #pragma unroll
-      for (int e = 0; e < kE; ++e) {
-        float a = acc[e];
+      for (int v = 0; v < kV; ++v) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) a = fmaf(pz[u], sV[kk + u][kSimtParts * e + part], a);
-        acc[e] = a;
+        for (int u = 0; u < 4; ++u) {
+          const float4 vx = reinterpret_cast<const float4*>(sV[kk + u])[4 * v + part];
+          acc[v].x = fmaf(pz[u], vx.x, acc[v].x);
+          acc[v].y = fmaf(pz[u], vx.y, acc[v].y);
+          acc[v].z = fmaf(pz[u], vx.z, acc[v].z);
+          acc[v].w = fmaf(pz[u], vx.w, acc[v].w);
+        }
       }
     }
   }
@@ -177,21 +206,26 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
 #pragma unroll
   for (int half = 2; half >= 1; half >>= 1) {
     if (grp >= half && grp < 2 * half) {
-      float* slot = grp == half ? &sK[0][0] : &sV[0][0];
+      float4* slot = reinterpret_cast<float4*>(grp == half ? &sK[0][0] : &sV[0][0]);
 #pragma unroll
-      for (int e = 0; e < kE; ++e) slot[t * D + kSimtParts * e + part] = acc[e];
+      for (int v = 0; v < kV; ++v) slot[t * (D / 4) + 4 * v + part] = acc[v];
     }
     __syncthreads();
     if (grp < half) {
-      const float* slot = grp == 0 ? &sK[0][0] : &sV[0][0];
+      const float4* slot = reinterpret_cast<const float4*>(grp == 0 ? &sK[0][0] : &sV[0][0]);
       const float mo = s_m[grp + half][t], lo = s_l[grp + half][t];
       const float mn = fmaxf(m, mo);
       const float a = (m == -INFINITY) ? 0.f : expf(m - mn);
       const float b = (mo == -INFINITY) ? 0.f : expf(mo - mn);
       l = l * a + lo * b;
 #pragma unroll
-      for (int e = 0; e < kE; ++e)
-        acc[e] = acc[e] * a + slot[t * D + kSimtParts * e + part] * b;
+      for (int v = 0; v < kV; ++v) {
+        const float4 o = slot[t * (D / 4) + 4 * v + part];
+        acc[v].x = acc[v].x * a + o.x * b;
+        acc[v].y = acc[v].y * a + o.y * b;
+        acc[v].z = acc[v].z * a + o.z * b;
+        acc[v].w = acc[v].w * a + o.w * b;
+      }
       m = mn;
     }
     __syncthreads();
@@ -204,7 +238,9 @@ __global__ void __launch_bounds__(kSimtThreads) attn_simt(const __grid_constant_
   if (live && grp == 0) {
     const float inv_l = 1.0f / l;
 #pragma unroll
-    for (int e = 0; e < kE; ++e) O[qoff + kSimtParts * e] = acc[e] * inv_l;
+    for (int v = 0; v < kV; ++v)
+      reinterpret_cast<float4*>(O)[qoff4 + 4 * v] =
+          make_float4(acc[v].x * inv_l, acc[v].y * inv_l, acc[v].z * inv_l, acc[v].w * inv_l);
   }
 }
 
