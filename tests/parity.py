@@ -18,12 +18,16 @@ ATT_MEAN_ABS = 1e-2
 
 
 def att_tol(wl, layer=0) -> float:
-    """Max-abs tolerance for bf16 attention. Rounding to bf16 (8 significant bits) moves a
-    value by at most 2^-8 of itself. The P weights go into the PV product rounded while the
-    fp32 row sum adds them unrounded: at most 2^-8 max|V| on the output; the output's own
-    rounding adds 2^-8 |O|; fp32 accumulation and the exp2 approximation stay far below.
-    With |O| <= max|V| the error is at most 2^-7 max|V|; the tolerance is 2.25 times that,
-    and never less than the 2e-2 of the stated workloads (whose outputs are far below 1)."""
+    """Max-abs tolerance for bf16 attention. Rounding to bf16 (8 significant bits, u = 2^-8)
+    moves a value by at most u of itself. The P weights enter the PV product rounded and the
+    fp32 row sum adds the same rounded weights, so the output is a convex combination of V
+    rows whose weights w~_i = w_i (1 + e_i) / (1 + sum_j w_j e_j) differ from the exact w_i
+    by at most 2u / (1 - u) of themselves; since the weight changes sum to zero, the output
+    moves by at most that times max_i |v_i - c| for c the midpoint of the values, i.e. by
+    about 2^-7 max|V|. The output's own rounding adds u |O| <= 2^-8 max|V|; fp32
+    accumulation and the exp2 approximation stay far below. The tolerance is 2.25 2^-7
+    max|V| (above that 1.5 2^-7 bound), and never less than the 2e-2 of the stated
+    workloads (whose outputs are far below 1)."""
     vmax = float(np.abs(wl.v[layer]).max()) if len(wl.v) else 0.0
     return max(ATT_MAX_ABS, 2.25 * 2.0 ** -7 * vmax)
 

@@ -154,6 +154,42 @@ def test_mask_probe_uniform_states(states, tc):
     assert mx <= _probe_tol(wl)
 
 
+@pytest.mark.parametrize("case", range(6))
+def test_attention_fp32_random_shapes(case):
+    """The fp32 CUDA-core kernel on seeded random ragged batches: sequences down to one row
+    (key groups that see no key merge as empty), blocks anywhere, S = 0, grouped heads,
+    both head dims, random query starts and score scales. fp32 throughout."""
+    rng = np.random.default_rng(700 + case)
+    specs = []
+    for _ in range(int(rng.integers(1, 5))):
+        n = int(rng.integers(1, 300))
+        B_ = int(rng.integers(0, min(n, 64) + 1))
+        b0 = int(rng.integers(0, n - B_ + 1))
+        shadow = ["paper", "candidates", "none"][int(rng.integers(0, 3))]
+        sp = dict(n_orig=n, block_start=b0, block_len=B_,
+                  fractions=tuple(rng.dirichlet([1, 1, 1])))
+        sp["shadow"] = np.zeros(0, np.int32) if shadow == "none" else shadow
+        if rng.random() < 0.4:
+            sp["query_start"] = int(rng.integers(0, n + 1))
+        specs.append(sp)
+    # a sequence of one to five rows: most key groups of its CTAs see no key
+    specs.append(dict(n_orig=int(rng.integers(1, 6)), block_start=0, block_len=1,
+                      fractions=(0.4, 0.3, 0.3)))
+    hkv = int(rng.choice([1, 2]))
+    hq = hkv * int(rng.choice([1, 3]))
+    d = int(rng.choice([64, 128]))
+    wl = W.custom(specs, hq, hkv, d, dtype="f32", seed=750 + case, qkv_std=float(rng.choice([0.2, 1.0])))
+    scale = float(rng.choice([0.0, 0.3, 1.0]))
+    ds, o = _attend(wl, scale=scale)
+    if any(sq.query_start < sq.rows for sq in wl.seqs):
+        mx, mean, n = P.compare_attention(wl, 0, o, scale=scale or None)
+        vmax = max(1.0, float(np.abs(wl.v[0]).max()))
+        print("fp32 random", case, [(sq.n_orig, sq.block_len, sq.n_shadow, sq.query_start)
+                                    for sq in wl.seqs], hq, hkv, d, scale, mx, mean)
+        assert mx <= 2e-4 * vmax
+    assert int(ds.status.item()) == 0
+
+
 @pytest.mark.parametrize("case", range(12))
 def test_attention_random_shapes(case, tc):
     """Seeded random ragged batches: odd lengths, blocks at the start / end, S = 0,
