@@ -23,12 +23,13 @@
 //   bandwidth goes to K and V only.
 //
 // attn_tc2: two 128-row query tiles of the same (sequence, head), so that every K/V tile
-// serves 256 rows; 11 warps:
+// serves 256 rows; 12 warps (warp 11 spare: it completes the side warpgroup's register split):
 //   warps 4q .. 4q + 3  softmax and epilogue of tile q, one thread per query row;
 //   warp 8              TMA producer: both Q tiles, then K and V through 2 stages each;
 //   warp 9              TMEM allocator and S issuer: S_q(j) = Q_q K(j)^T (Q from shared
 //                       memory), once PV_q(j - 1) has read P_q(j - 1) out of S_q's columns;
-//   warp 10             PV issuer: O_q += P_q(j) V(j) once P_q(j) is stored.
+//   warp 10             PV issuer: O_q += P_q(j) V(j), each 64-key half as soon as that half
+//                       of P_q(j) is stored.
 //   TMEM: S_0, S_1 [0, 256) with P_q(j) written over the first 64 columns of S_q(j),
 //   O_0, O_1 [256, 256 + 2D).
 // Both keep a per-row running maximum and rescale O in TMEM only when the maximum grows by
@@ -512,14 +513,15 @@ __device__ __forceinline__ float tile_row_load(uint32_t tS, uint64_t vis0, uint6
   return fmaxf(fmax3(mx[0], mx[1], mx[2]), fmax3(fmax3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
 }
 
-// P = 2^(s * sl - mL) for the row's 128 scores held in registers, stored as bf16 pairs over
-// columns tS .. tS + 63 (the first half of the S tile's columns); the stored (rounded) values
-// are summed into acc (four packed partial sums), so that the output is a convex combination
-// of V rows with exactly the weights the PV product uses.
+// P = 2^(s * sl - mL) for keys 64 hh .. 64 hh + 63 of the row's 128 scores held in
+// registers, stored as bf16 pairs over columns tS + 32 hh .. tS + 32 hh + 31 (in the first
+// half of the S tile's columns); the stored (rounded) values are summed into acc (four packed
+// partial sums), so that the output is a convex combination of V rows with exactly the
+// weights the PV product uses.
+template <int hh>
 __device__ __forceinline__ void tile_row_exp(uint32_t tS, const uint32_t (&sv)[128],
                                              uint64_t sl2, uint64_t nmL2, uint64_t (&acc)[4]) {
-#pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
+  {
     uint32_t pk[32];
 #pragma unroll
     for (int e = 0; e < 32; ++e) {
@@ -545,7 +547,7 @@ struct __align__(16) Tc2Ctl {
   uint64_t q_rot[kQT];   // RoPE: the softmax warps of tile q rotated it in shared memory
   uint64_t k_full[kNK], k_empty[kNK], v_full[kNV], v_empty[kNV];
   uint64_t s_full[kQT];   // S_q(j) landed in TMEM
-  uint64_t p_full[kQT];   // the softmax of tile q stored P_q(j) over S_q(j)
+  uint64_t p_half[kQT][2];  // the softmax of tile q stored keys 64 h .. 64 h + 63 of P_q(j)
   uint64_t pv_done[kQT];  // PV_q(j) completed: S_q's columns may take S_q(j + 1)
   uint64_t o_full[kQT];   // the last PV_q completed
   uint64_t drained;       // every product both issuers launched has completed (two commits)
@@ -632,7 +634,8 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     }
     for (int q = 0; q < kQT; ++q) {
       mbar_init(&ctl.s_full[q], 1);
-      mbar_init(&ctl.p_full[q], 4);
+      mbar_init(&ctl.p_half[q][0], 4);
+      mbar_init(&ctl.p_half[q][1], 4);
       mbar_init(&ctl.pv_done[q], 1);
       mbar_init(&ctl.o_full[q], 1);
     }
@@ -748,7 +751,9 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   } else if (warp == kWPv) {
     // ------------------------------------------------------------ PV issuer
     reg_dealloc<kTc2SideRegs>();
-    // O_q += P_q(j) V(j) once the softmax of tile q has stored P_q(j) and V(j) has landed.
+    // O_q += P_q(j) V(j) once V(j) has landed, in two halves of 64 keys: each as soon as
+    // the softmax of tile q has stored that half of P_q(j), so that the first half's
+    // products run while the softmax computes the second.
     if (lane == 0) {
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, 0, 1);
       const uint32_t av = smem_u32(sV);
@@ -756,15 +761,19 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       for (int j = 0; j < n_kt && ok && !*abort_flag; ++j) {
         ok = mbar_wait(&ctl.v_full[j % kNV], (j / kNV) & 1, wlim);
         for (int q = 0; q < nq && ok; ++q) {
-          ok = mbar_wait(&ctl.p_full[q], j & 1, wlim);
-          if (!ok) break;
-          tc_fence_after();
           const uint32_t vaddr = av + (j % kNV) * kTileBytes;
 #pragma unroll
-          for (int ks = 0; ks < kTN / 16; ++ks)
-            mma_ts(tO0 + q * D, tS0 + q * kTN + ks * 8,
-                   smem_desc_sw128(vaddr + ks * 2048, kKSub, 1024), kIdO,
-                   (j > 0 || ks > 0) ? 1u : 0u);
+          for (int hh = 0; hh < 2; ++hh) {
+            ok = ok && mbar_wait(&ctl.p_half[q][hh], j & 1, wlim);
+            if (!ok) break;
+            tc_fence_after();
+#pragma unroll
+            for (int ks = 4 * hh; ks < 4 * hh + 4; ++ks)
+              mma_ts(tO0 + q * D, tS0 + q * kTN + ks * 8,
+                     smem_desc_sw128(vaddr + ks * 2048, kKSub, 1024), kIdO,
+                     (j > 0 || ks > 0) ? 1u : 0u);
+          }
+          if (!ok) break;
           mma_commit(&ctl.pv_done[q]);
           if (j == n_kt - 1) mma_commit(&ctl.o_full[q]);
         }
@@ -835,7 +844,13 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       // P over the first 64 columns of S_q(j), and the row sum
       const uint64_t sl2 = f2_pack(sl, sl), nmL2 = f2_pack(-mL, -mL);
       uint64_t acc[4] = {0, 0, 0, 0};  // bit pattern 0 = +0.0f
-      tile_row_exp(tS + lane_off, sv, sl2, nmL2, acc);
+      // the first half of P, handed to the PV issuer before the second is computed
+      tile_row_exp<0>(tS + lane_off, sv, sl2, nmL2, acc);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.p_half[q][0]);
+      tile_row_exp<1>(tS + lane_off, sv, sl2, nmL2, acc);
       float a0, a1, b0, b1;
       f2_unpack(f2_add(acc[0], acc[1]), a0, a1);
       f2_unpack(f2_add(acc[2], acc[3]), b0, b1);
@@ -844,7 +859,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.p_full[q]);
+      if (lane == 0) mbar_arrive(&ctl.p_half[q][1]);
     }
     if (active) {
       if (ok) ok = mbar_wait(&ctl.o_full[q], 0, wlim);
