@@ -12,12 +12,14 @@ namespace {
 // row in each of four key groups, 512 threads: thread `part` of a row owns the four-element
 // vectors 16 v + 4 part .. 16 v + 4 part + 3 (v = 0 .. D/16 - 1) of q and of its O
 // accumulator, so that the row's four threads read 64 contiguous bytes of a shared-memory
-// key row per vector (one 16-byte load each, no bank conflict). The sequence's keys pass through shared
-// memory 32 rows at a time (K and V, read as broadcasts); key group `grp` takes keys
-// 8 grp .. 8 grp + 7 of every tile, four at a time: four independent partial dot products,
-// which the row's four threads add up with two shuffles each, then one online softmax step
-// over the four. At the end the four groups' (maximum, sum, accumulator) of a row are
-// merged through shared memory. Masking as on the tensor-core path, by key_visible().
+// key row per vector (one 16-byte load each, no bank conflict). The sequence's keys pass
+// through shared memory 32 rows at a time (K and V, read as broadcasts; each thread loads
+// its share of the next tile while the current one is computed); key group `grp` takes
+// keys 8 grp .. 8 grp + 7 of every tile, four at a time: four independent partial dot
+// products, which the row's four threads add up with two shuffles each, then one online
+// softmax step over the four. At the end the four groups' (maximum, sum, accumulator) of a
+// row are merged through shared memory. Masking as on the tensor-core path, by
+// key_visible().
 constexpr int kSimtRows = 32;     // query rows per CTA
 constexpr int kSimtParts = 4;     // threads per query row and key group
 constexpr int kSimtGroups = 4;    // key groups
